@@ -1,0 +1,375 @@
+/*
+ * Oracle (test infrastructure only): the compressed state of one head and the
+ * persistent decode step (App. C.3, "One persistent STEPQuant decode step").
+ *
+ * Representation (Sec. 4.3): X_hat_ij = r_i c_j z_ij with FP16 row factors r,
+ * FP16 column factors c and integer codes. Head units (GDN) use z = q with
+ * |q| <= 2^(b-1)-1 (Eq. uniform_quantization). Row units (KDA) use the
+ * normalised codebook z = 2^(8-b_i) q (App. C.1), so rows of different widths
+ * share one column vector. FP16 pivots store X directly (Sec. 3.2).
+ *
+ * Readings where the paper is silent (listed in the design notes):
+ *  - r_i = fp16(clamp(sqrt(m_i) * w_i^(-1/2), 2^-14, 65504)), the FP16 clamp of
+ *    the baseline's scale storage (App. B.5);
+ *  - the column fit starts from the clip-free value
+ *    c0_j = max_{i in I} |X_ij| / (r_i zs_i qmax_i), then applies `fit_iters`
+ *    fixed-code updates c_j = sum w_i^2 v_ij X_ij / sum w_i^2 v_ij^2 (App. C.1),
+ *    a zero denominator keeping the current iterate, floor 2^-14, cap 65504;
+ *  - "round to the nearest level" is round-half-to-even of the fp32 value
+ *    t = fp32(fp32(X * rho_i) * gamma_j), rho_i = fp32(1/(r_i zs_i)),
+ *    gamma_j = fp32(1/c_j): the decision is taken in the GPU tile's precision;
+ *  - codes are stored offset-binary u = q + 2^(b-1), LSB-first per row.
+ *
+ * Page layout of one head (all pieces 16-byte multiples):
+ *   integer head unit: r[128] fp16 | c[128] fp16 | 128 rows x 16b bytes
+ *   pivot head unit:   128 rows x 256 bytes (fp16 values)
+ *   row-unit head:     r[128] fp16 | c[128] fp16 | row i: 16 b_i bytes
+ *                      (b_i = 16 marks an FP16 pivot row, 256 bytes)
+ */
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+#include "oracle.h"
+
+#define F16_MIN_NORMAL (1.0 / 16384.0)   /* 2^-14 */
+#define F16_MAX 65504.0
+
+static int is_pivot_head(int unit_kind, const int8_t *rb)
+{
+    return unit_kind == OR_UNIT_HEAD && rb[0] == OR_PIVOT_BITS;
+}
+
+static int qmax_of(int b) { return (1 << (b - 1)) - 1; }
+
+/* codebook spacing: 2^(8-b) for the normalised row-unit codebook, 1 otherwise */
+static int zs_of(int unit_kind, int b) { return unit_kind == OR_UNIT_ROW ? 1 << (8 - b) : 1; }
+
+static double clampd(double x, double lo, double hi) { return x < lo ? lo : (x > hi ? hi : x); }
+
+/* fp32 product of two fp32 values (exact in fp64, rounded once) */
+static float mul32(float a, float b) { return (float)((double)a * (double)b); }
+
+size_t or_head_bytes(int unit_kind, const int8_t *rb)
+{
+    if (is_pivot_head(unit_kind, rb))
+        return (size_t)OR_D * 256;
+    size_t n = 512;
+    for (int i = 0; i < OR_D; i++)
+        n += 16 * (size_t)rb[i];
+    return n;
+}
+
+static size_t row_offset(int unit_kind, const int8_t *rb, int i)
+{
+    if (is_pivot_head(unit_kind, rb))
+        return (size_t)i * 256;
+    size_t off = 512;
+    for (int t = 0; t < i; t++)
+        off += 16 * (size_t)rb[t];
+    return off;
+}
+
+static void put_u16(uint8_t *p, uint16_t v) { p[0] = v & 0xFF; p[1] = v >> 8; }
+static uint16_t get_u16(const uint8_t *p) { return (uint16_t)(p[0] | (p[1] << 8)); }
+
+/* Write code u (b bits) at bit position pos of a little-endian bit stream. */
+static void put_bits(uint8_t *row, int pos, int b, unsigned u)
+{
+    for (int t = 0; t < b; t++) {
+        int p = pos + t;
+        if ((u >> t) & 1u)
+            row[p >> 3] |= (uint8_t)(1u << (p & 7));
+        else
+            row[p >> 3] &= (uint8_t)~(1u << (p & 7));
+    }
+}
+
+static unsigned get_bits(const uint8_t *row, int pos, int b)
+{
+    unsigned u = 0;
+    for (int t = 0; t < b; t++) {
+        int p = pos + t;
+        u |= (unsigned)((row[p >> 3] >> (p & 7)) & 1u) << t;
+    }
+    return u;
+}
+
+/* Unpack a head page into scales, integer codes and pivot values. For a
+ * pivot head r and c are zero and every row is in `piv`. */
+void or_unpack_head(const uint8_t *page, int unit_kind, const int8_t *rb,
+                    uint16_t *r, uint16_t *c, int8_t *codes, uint16_t *piv)
+{
+    int ph = is_pivot_head(unit_kind, rb);
+    for (int i = 0; i < OR_D; i++) {
+        r[i] = ph ? 0 : get_u16(page + 2 * i);
+        c[i] = ph ? 0 : get_u16(page + 256 + 2 * i);
+    }
+    for (int i = 0; i < OR_D; i++) {
+        const uint8_t *row = page + row_offset(unit_kind, rb, i);
+        int b = rb[i];
+        for (int j = 0; j < OR_D; j++) {
+            if (b == OR_PIVOT_BITS) {
+                piv[i * OR_D + j] = get_u16(row + 2 * j);
+                codes[i * OR_D + j] = 0;
+            } else {
+                unsigned u = get_bits(row, j * b, b);
+                codes[i * OR_D + j] = (int8_t)((int)u - (1 << (b - 1)));
+                piv[i * OR_D + j] = 0;
+            }
+        }
+    }
+}
+
+/* Reconstruction (App. C.3 step 1): S_ij = r_i c_j z_ij, or the FP16 value for
+ * pivot units. Exact in fp64. */
+void or_decode_head(const uint8_t *page, int unit_kind, const int8_t *rb, double *S)
+{
+    uint16_t r[OR_D], c[OR_D];
+    int8_t *codes = malloc(OR_N);
+    uint16_t *piv = malloc(sizeof(uint16_t) * OR_N);
+    or_unpack_head(page, unit_kind, rb, r, c, codes, piv);
+    for (int i = 0; i < OR_D; i++) {
+        int b = rb[i];
+        for (int j = 0; j < OR_D; j++) {
+            if (b == OR_PIVOT_BITS)
+                S[i * OR_D + j] = or_fp16_decode(piv[i * OR_D + j]);
+            else
+                S[i * OR_D + j] = or_fp16_decode(r[i]) * or_fp16_decode(c[j]) *
+                                  (double)zs_of(unit_kind, b) * (double)codes[i * OR_D + j];
+        }
+    }
+    free(codes);
+    free(piv);
+}
+
+void or_decode_head_f32(const uint8_t *page, int unit_kind, const int8_t *rb, float *S)
+{
+    double *D = malloc(sizeof(double) * OR_N);
+    or_decode_head(page, unit_kind, rb, D);
+    for (int t = 0; t < OR_N; t++)
+        S[t] = (float)D[t];
+    free(D);
+}
+
+/* Key-Row-Aware Dual-axis Fitting of an updated tile X (fp32, row-major)
+ * (Sec. 4.3; App. C.1; App. C.3 steps 4-5). Outputs the FP16 row factors r,
+ * the per-row reciprocal rho_i = fp32(1/(r_i zs_i)), the final fp32 column
+ * iterate and the codes of the last fixed-code update (for inspection). */
+static void fit_head(const float *X, int unit_kind, const int8_t *rb, const float *w,
+                     int fit_iters, double *r, float *rho, float *c, int8_t *z_last)
+{
+    float rho_max[OR_D];      /* fp32(1 / (r_i zs_i qmax_i)) */
+    int in_fit[OR_D];         /* non-pivot integer rows: the set I */
+    for (int i = 0; i < OR_D; i++) {
+        int b = rb[i];
+        in_fit[i] = (b != OR_PIVOT_BITS);
+        if (!in_fit[i]) {
+            r[i] = 0.0;
+            rho[i] = rho_max[i] = 0.0f;
+            continue;
+        }
+        /* Row factors: m_i = (1/d_v) sum_j |X_ij|, r_i = m_i^(1/2) w_i^(-1/2). */
+        double s = 0.0;
+        for (int j = 0; j < OR_D; j++)
+            s += fabs((double)X[i * OR_D + j]);
+        float m = (float)(s / OR_D);
+        float wis = (float)(1.0 / sqrt((double)w[i]));
+        float t = mul32(sqrtf(m), wis);
+        r[i] = or_fp16_round(clampd(t, F16_MIN_NORMAL, F16_MAX));
+        double zs = zs_of(unit_kind, b);
+        rho[i] = (float)(1.0 / (r[i] * zs));
+        rho_max[i] = (float)(1.0 / (r[i] * zs * qmax_of(b)));
+    }
+    /* Column factors: clip-free start, then fixed-code least-squares updates of
+     * min_c sum_ij w_i^2 (X_ij - r_i c_j z_ij)^2 over the rows in I. */
+    for (int j = 0; j < OR_D; j++) {
+        float cmax = 0.0f;
+        for (int i = 0; i < OR_D; i++)
+            if (in_fit[i]) {
+                float a = mul32(fabsf(X[i * OR_D + j]), rho_max[i]);
+                if (a > cmax)
+                    cmax = a;
+            }
+        c[j] = (float)clampd(cmax, F16_MIN_NORMAL, F16_MAX);
+    }
+    if (z_last)
+        for (int t = 0; t < OR_N; t++)
+            z_last[t] = 0;
+    for (int it = 0; it < fit_iters; it++) {
+        for (int j = 0; j < OR_D; j++) {
+            float gamma = (float)(1.0 / (double)c[j]);
+            double num = 0.0, den = 0.0;
+            for (int i = 0; i < OR_D; i++) {
+                if (!in_fit[i])
+                    continue;
+                int b = rb[i], qm = qmax_of(b);
+                float t = mul32(mul32(X[i * OR_D + j], rho[i]), gamma);
+                double qv = clampd(rint((double)t), -qm, qm);
+                if (z_last)
+                    z_last[i * OR_D + j] = (int8_t)qv;
+                double v = r[i] * (double)zs_of(unit_kind, b) * qv;      /* v_ij = r_i z_ij */
+                double w2 = (double)w[i] * (double)w[i];
+                num += w2 * v * (double)X[i * OR_D + j];
+                den += w2 * v * v;
+            }
+            if (den > 0.0)
+                c[j] = (float)clampd((double)(float)(num / den), F16_MIN_NORMAL, F16_MAX);
+        }
+    }
+}
+
+void or_fit_debug(const float *X, int unit_kind, const int8_t *rb, const float *w,
+                  int fit_iters, double *r, float *c_iter, int8_t *z_last)
+{
+    float rho[OR_D];
+    fit_head(X, unit_kind, rb, w, fit_iters, r, rho, c_iter, z_last);
+}
+
+/* Fit, then pack with the stored FP16 scales (App. C.3 step 6). */
+void or_encode_head(const float *X, int unit_kind, const int8_t *rb, const float *w,
+                    int fit_iters, uint8_t *page)
+{
+    if (is_pivot_head(unit_kind, rb)) {             /* FP16 pivot head */
+        for (int i = 0; i < OR_D; i++)
+            for (int j = 0; j < OR_D; j++)
+                put_u16(page + (size_t)i * 256 + 2 * j,
+                        or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
+        return;
+    }
+    double r[OR_D];
+    float rho[OR_D], c[OR_D];
+    fit_head(X, unit_kind, rb, w, fit_iters, r, rho, c, NULL);
+    /* Storage precision and final codes with the stored scales. */
+    double c16[OR_D];
+    float gamma[OR_D];
+    for (int j = 0; j < OR_D; j++) {
+        c16[j] = or_fp16_round(c[j]);
+        gamma[j] = (float)(1.0 / c16[j]);
+    }
+    for (int i = 0; i < OR_D; i++) {
+        put_u16(page + 2 * i, or_fp16_encode(r[i]));
+        put_u16(page + 256 + 2 * i, or_fp16_encode(c16[i]));
+    }
+    for (int i = 0; i < OR_D; i++) {
+        uint8_t *row = page + row_offset(unit_kind, rb, i);
+        int b = rb[i];
+        if (b == OR_PIVOT_BITS) {
+            for (int j = 0; j < OR_D; j++)
+                put_u16(row + 2 * j, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
+            continue;
+        }
+        int qm = qmax_of(b);
+        for (int j = 0; j < OR_D; j++) {
+            float t = mul32(mul32(X[i * OR_D + j], rho[i]), gamma[j]);
+            int qv = (int)clampd(rint((double)t), -qm, qm);
+            put_bits(row, j * b, b, (unsigned)(qv + (1 << (b - 1))));
+        }
+    }
+}
+
+/* One persistent decode step of one head (App. C.3 steps 1-7): reconstruct,
+ * X = D S + beta k (v^T - k^T D S), y = X^T q, refit, requantize in place. */
+void or_step_head(uint8_t *page, int unit_kind, const int8_t *rb, const float *w,
+                  int fit_iters, const float *q, const float *k, const float *v,
+                  float beta, const float *gate, int gate_per_row, float *y)
+{
+    double *S = malloc(sizeof(double) * OR_N);
+    float *X = malloc(sizeof(float) * OR_N);
+    double u[OR_D];
+    or_decode_head(page, unit_kind, rb, S);
+    for (int i = 0; i < OR_D; i++) {
+        double d = gate_per_row ? gate[i] : gate[0];
+        for (int j = 0; j < OR_D; j++)
+            S[i * OR_D + j] *= d;                              /* D S_hat */
+    }
+    for (int j = 0; j < OR_D; j++) {
+        double acc = 0.0;
+        for (int i = 0; i < OR_D; i++)
+            acc += (double)k[i] * S[i * OR_D + j];
+        u[j] = acc;
+    }
+    for (int i = 0; i < OR_D; i++)
+        for (int j = 0; j < OR_D; j++)
+            X[i * OR_D + j] = (float)(S[i * OR_D + j] +
+                                      (double)beta * (double)k[i] * ((double)v[j] - u[j]));
+    for (int j = 0; j < OR_D; j++) {                           /* readout before requantization */
+        double acc = 0.0;
+        for (int i = 0; i < OR_D; i++)
+            acc += (double)q[i] * (double)X[i * OR_D + j];
+        y[j] = (float)acc;
+    }
+    or_encode_head(X, unit_kind, rb, w, fit_iters, page);
+    free(S);
+    free(X);
+}
+
+/* ---- uniform rowwise-absmax INT-b baseline ----
+ * Every key row uses the scale s_i = absmax_i / qmax stored in FP16, clamped
+ * to [2^-14, 65504], and nearest-integer codes in [-qmax, qmax] (App. B.5).
+ * Page: s[128] fp16 | 128 rows x 16b bytes (offset-binary codes, LSB-first).
+ * The code decision uses t = fp32(X * fp32(1/s_i)). */
+size_t or_intb_head_bytes(int bits) { return 256 + (size_t)OR_D * 16 * bits; }
+
+void or_intb_encode_head(const float *X, int bits, uint8_t *page)
+{
+    int qm = qmax_of(bits);
+    for (int i = 0; i < OR_D; i++) {
+        float amax = 0.0f;
+        for (int j = 0; j < OR_D; j++)
+            if (fabsf(X[i * OR_D + j]) > amax)
+                amax = fabsf(X[i * OR_D + j]);
+        float s = (float)((double)amax / qm);
+        double s16 = or_fp16_round(clampd(s, F16_MIN_NORMAL, F16_MAX));
+        float inv = (float)(1.0 / s16);
+        put_u16(page + 2 * i, or_fp16_encode(s16));
+        uint8_t *row = page + 256 + (size_t)i * 16 * bits;
+        for (int j = 0; j < OR_D; j++) {
+            float t = mul32(X[i * OR_D + j], inv);
+            int qv = (int)clampd(rint((double)t), -qm, qm);
+            put_bits(row, j * bits, bits, (unsigned)(qv + (1 << (bits - 1))));
+        }
+    }
+}
+
+void or_intb_decode_head(const uint8_t *page, int bits, double *S)
+{
+    for (int i = 0; i < OR_D; i++) {
+        double s = or_fp16_decode(get_u16(page + 2 * i));
+        const uint8_t *row = page + 256 + (size_t)i * 16 * bits;
+        for (int j = 0; j < OR_D; j++)
+            S[i * OR_D + j] = s * (double)((int)get_bits(row, j * bits, bits) - (1 << (bits - 1)));
+    }
+}
+
+void or_intb_step_head(uint8_t *page, int bits, const float *q, const float *k, const float *v,
+                       float beta, const float *gate, int gate_per_row, float *y)
+{
+    double *S = malloc(sizeof(double) * OR_N);
+    float *X = malloc(sizeof(float) * OR_N);
+    double u[OR_D];
+    or_intb_decode_head(page, bits, S);
+    for (int i = 0; i < OR_D; i++) {
+        double d = gate_per_row ? gate[i] : gate[0];
+        for (int j = 0; j < OR_D; j++)
+            S[i * OR_D + j] *= d;
+    }
+    for (int j = 0; j < OR_D; j++) {
+        double acc = 0.0;
+        for (int i = 0; i < OR_D; i++)
+            acc += (double)k[i] * S[i * OR_D + j];
+        u[j] = acc;
+    }
+    for (int i = 0; i < OR_D; i++)
+        for (int j = 0; j < OR_D; j++)
+            X[i * OR_D + j] = (float)(S[i * OR_D + j] +
+                                      (double)beta * (double)k[i] * ((double)v[j] - u[j]));
+    for (int j = 0; j < OR_D; j++) {
+        double acc = 0.0;
+        for (int i = 0; i < OR_D; i++)
+            acc += (double)q[i] * (double)X[i * OR_D + j];
+        y[j] = (float)acc;
+    }
+    or_intb_encode_head(X, bits, page);
+    free(S);
+    free(X);
+}

@@ -1,0 +1,157 @@
+"""Pins of the oracle's offline plan: row-impact factors (Sec. 4.3 footnote),
+lifetime weights (Eq. calibration_lifetime), the allocation optimisers
+(Eq. allocation, App. C.2), FP16 pivots and the packed byte counts the paper
+prints (App. D, App. F.1; fixtures in tests/golden/storage.json).
+"""
+import itertools
+import json
+import os
+
+import numpy as np
+import pytest
+
+D = 128
+HEAD, ROW = 0, 1
+GOLD = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "storage.json")))
+
+
+def test_row_weights_geometric_mean_and_ratios(oracle, rng):
+    omega = np.exp(rng.normal(0, 3, (3, D))).astype(np.float32)
+    w = oracle.row_weights(omega)
+    for h in range(3):
+        assert abs(np.mean(np.log(w[h].astype(np.float64)))) < 1e-6       # GM(w) = 1
+        i, k = rng.choice(D, 2, replace=False)
+        ratio = (w[h, i] / w[h, k]).astype(np.float64) ** 8                 # w ~ omega^(gamma/2)
+        assert abs(ratio / (omega[h, i] / omega[h, k]) - 1) < 1e-5
+
+
+def test_lifetime_weight_closed_form(oracle):
+    for ell in (-0.5, -0.05, -1e-3, -1e-6):
+        for H in (1, 7, 2048):
+            ref = (1 - np.exp(2 * H * ell)) / (1 - np.exp(2 * ell))
+            assert abs(oracle.lifetime_weight(ell, H) - ref) <= 1e-9 * ref
+    assert oracle.lifetime_weight(0.0, 100) == 100
+
+
+def _brute(cost, cands, fits):
+    U, K = cost.shape
+    best, arg = np.inf, None
+    for ch in itertools.product(range(K), repeat=U):
+        if not fits(sum(cands[k] for k in ch)):
+            continue
+        val = sum(cost[u, k] for u, k in enumerate(ch))
+        if val < best:
+            best, arg = val, ch
+    return best, arg
+
+
+def _random_costs(rng, U, cands):
+    d = np.sort(np.exp(rng.normal(0, 2, (U, len(cands)))), axis=1)[:, ::-1]   # decreasing in b
+    return d * np.exp(rng.normal(0, 1, (U, 1)))
+
+
+@pytest.mark.parametrize("cands", [(4, 6, 8), (2, 4, 6, 8)])
+def test_dp_equals_brute_force(oracle, rng, cands):
+    for _ in range(25):
+        U = int(rng.integers(1, 7))
+        cost = _random_costs(rng, U, cands)
+        cap = int(rng.integers(min(cands) // 2 * U, max(cands) // 2 * U + 1))
+        ch = oracle.allocate_dp(cost, cands, cap)
+        best, _ = _brute(cost, cands, lambda bits: bits <= 2 * cap)
+        assert ch is not None
+        assert sum(cands[k] for k in ch) <= 2 * cap
+        assert abs(sum(cost[u, k] for u, k in enumerate(ch)) - best) <= 1e-12 * best
+    assert oracle.allocate_dp(np.ones((3, 3)), (4, 6, 8), 5) is None          # 3 units need >= 6
+
+
+@pytest.mark.parametrize("cands", [(4, 6, 8), (2, 4, 6, 8)])
+def test_lagrangian_feasible_and_near_optimal(oracle, rng, cands):
+    excess = []
+    for _ in range(25):
+        U = int(rng.integers(2, 7))
+        cost = _random_costs(rng, U, cands)
+        budget = int(rng.integers(min(cands) * U, max(cands) * U + 1))
+        ch = oracle.allocate_lagrangian(cost, cands, budget)
+        best, _ = _brute(cost, cands, lambda bits: bits <= budget)
+        val = sum(cost[u, k] for u, k in enumerate(ch))
+        assert sum(cands[k] for k in ch) <= budget
+        assert val >= best * (1 - 1e-12)
+        assert val <= best + np.max(cost[:, 0] - cost[:, -1])
+        excess.append(val / best - 1)
+    assert np.median(excess) < 0.05
+    assert oracle.allocate_lagrangian(np.ones((3, 3)), (4, 6, 8), 11) is None
+
+
+def test_lagrangian_uses_whole_budget_when_everything_fits(oracle, rng):
+    cost = _random_costs(rng, 5, (2, 4, 6, 8))
+    ch = oracle.allocate_lagrangian(cost, (2, 4, 6, 8), 40)
+    assert all(k == 3 for k in ch)
+
+
+def test_head_pivots_rank_residual_risk(oracle, rng):
+    cands = (4, 6, 8)
+    U, nominal, n_piv = 6, 6, 2
+    dist = np.concatenate([_random_costs(rng, U, cands), 1e-9 * np.ones((U, 1))], axis=1)
+    L = np.exp(rng.normal(0, 1, U))
+    piv = oracle.select_pivots(HEAD, cands, nominal, L, dist, n_piv)
+    _, arg = _brute(L[:, None] * dist[:, :3], cands, lambda bits: bits <= nominal * U)
+    risk = np.array([L[u] * dist[u, k] for u, k in enumerate(arg)])
+    assert set(np.flatnonzero(piv)) == set(np.argsort(-risk, kind="stable")[:n_piv])
+    bits = oracle.allocate(HEAD, cands, nominal, L, dist, piv)
+    assert np.all(bits[piv == 1] == 16)
+    # pivots are 8-bit replacements against the nominal budget
+    assert np.sum(bits[piv == 0]) + 8 * n_piv <= nominal * U
+
+
+def test_row_pivots_rank_fp16_reduction(oracle, rng):
+    cands = (2, 4, 6, 8)
+    U = 40
+    dist = np.concatenate([_random_costs(rng, U, cands), np.exp(rng.normal(-12, 1, (U, 1)))], axis=1)
+    L = np.exp(rng.normal(0, 1, U))
+    piv = oracle.select_pivots(ROW, cands, 4, L, dist, 5)
+    risk = L * (dist[:, 1] - dist[:, 4])
+    assert set(np.flatnonzero(piv)) == set(np.argsort(-risk, kind="stable")[:5])
+    bits = oracle.allocate(ROW, cands, 4, L, dist, piv)
+    assert np.sum(bits[piv == 0]) + 8 * 5 <= 4 * U
+
+
+def _paper_plan(oracle, rng, g):
+    n_units = g["layers"] * g["heads"] * (1 if g["unit"] == "head" else D)
+    unit = HEAD if g["unit"] == "head" else ROW
+    cands = tuple(g["candidates"])
+    dist = np.concatenate([_random_costs(rng, n_units, cands),
+                           np.exp(rng.normal(-14, 1, (n_units, 1)))], axis=1)
+    L = np.exp(rng.normal(3, 1, n_units))
+    piv = oracle.select_pivots(unit, cands, g["nominal"], L, dist, g["pivots"])
+    bits = oracle.allocate(unit, cands, g["nominal"], L, dist, piv)
+    off, nb, stride = oracle.layout(unit, g["layers"], g["heads"], bits)
+    return unit, bits, off, nb, stride
+
+
+def test_qwen_at6_packed_bytes(oracle, rng):
+    """App. F.1: 29,999,104 B per request; App. F.3: 30,015,488 B with pivot scale
+    slots; Eq. compact_qwen: 6.3611 bits/value."""
+    g = GOLD["qwen_at6"]
+    unit, bits, off, nb, stride = _paper_plan(oracle, rng, g)
+    assert int(np.sum(bits == 16)) == g["pivots"]
+    total = int(np.sum(nb))
+    assert total == g["packed_bytes"] == stride
+    assert total + 512 * g["pivots"] == g["packed_bytes_with_pivot_scale_slots"]
+    N = g["layers"] * g["heads"] * D * D
+    assert 4 * N == g["fp32_bytes"]
+    assert round((total + 512 * g["pivots"]) * 8 / N, 4) == g["compact_bits"]
+    assert np.all(off % 16 == 0) and np.all(np.diff(off.astype(np.int64)) == nb[:-1])
+
+
+@pytest.mark.parametrize("key", ["kda_at6", "kda_at4"])
+def test_kda_packed_bytes(oracle, rng, key):
+    """App. D: KDA @6 = 7.875 MiB (6.30 bits/value), @4 = 5.375 MiB (4.30)."""
+    g = GOLD[key]
+    unit, bits, off, nb, stride = _paper_plan(oracle, rng, g)
+    total = int(np.sum(nb))
+    assert total == g["mib"] * 2 ** 20
+    N = g["layers"] * g["heads"] * D * D
+    assert round(total * 8 / N, 2) == g["compact_bits"]
+    if "fp32_mib" in g:
+        assert 4 * N == g["fp32_mib"] * 2 ** 20
+    assert stride % 256 == 0 and stride >= total

@@ -1,0 +1,125 @@
+"""Pins of the oracle's persistent decode step (App. C.3) and calibration drivers.
+
+* Steps 1-3: the readout is taken from the updated tile before requantization
+  (Eq. compressed_recurrence): it equals the FP32-state reference step applied
+  to the reconstructed state; with every unit an FP16 pivot the step is exactly
+  the FP32-state recurrence on FP16-rounded state.
+* Prop. 1: the readout error of the compressed path is (A_t E_{t-1})^T q_t.
+* Calibration (App. A.3): omega is the mean of g^2 with g = A^T q built densely.
+"""
+import numpy as np
+import pytest
+
+from paper_2609_38169_gb300 import workloads as W
+
+D = 128
+HEAD, ROW, PIV = 0, 1, 16
+
+
+def _inp(rng, per_row):
+    q = rng.standard_normal(D).astype(np.float32)
+    k = rng.standard_normal(D)
+    k = (k / np.linalg.norm(k)).astype(np.float32)
+    v = rng.standard_normal(D).astype(np.float32)
+    beta = np.float32(rng.uniform(0.1, 0.9))
+    gate = (rng.uniform(0.8, 0.999, D) if per_row else [rng.uniform(0.9, 0.999)])
+    return q, k, v, beta, np.asarray(gate, np.float32)
+
+
+def test_pivot_head_step_is_fp32_recurrence_on_fp16_state(oracle, rng):
+    S = (rng.standard_normal((D, D)) * 3).astype(np.float32)
+    rb = np.full(D, PIV, np.int8)
+    w = np.ones(D, np.float32)
+    page = oracle.encode_head(S, HEAD, rb, w)
+    S16 = oracle.decode_head_f32(page, HEAD, rb)
+    assert np.array_equal(S16, np.float16(S).astype(np.float32))
+    q, k, v, beta, gate = _inp(rng, False)
+    page1, y = oracle.step_head(page, HEAD, rb, w, q, k, v, beta, gate)
+    S1, yref = oracle.delta_step(S16, q, k, v, beta, gate)
+    assert np.array_equal(y, yref)
+    assert np.array_equal(oracle.decode_head_f32(page1, HEAD, rb), np.float16(S1).astype(np.float32))
+
+
+@pytest.mark.parametrize("unit", [HEAD, ROW])
+def test_step_reads_before_requantizing(oracle, rng, unit):
+    S = (rng.standard_normal((D, D)) * np.exp(rng.normal(size=(D, 1)))).astype(np.float32)
+    if unit == HEAD:
+        rb = np.full(D, 6, np.int8)
+    else:
+        rb = rng.choice([2, 4, 6, 8], D).astype(np.int8)
+        rb[:5] = PIV
+    w = np.exp(rng.normal(0, 0.3, D)).astype(np.float32)
+    page = oracle.encode_head(S, unit, rb, w)
+    q, k, v, beta, gate = _inp(rng, unit == ROW)
+    page1, y = oracle.step_head(page, unit, rb, w, q, k, v, beta, gate)
+    Shat = oracle.decode_head(page, unit, rb)
+    Dg = np.broadcast_to(gate.astype(np.float64), (D,))[:, None]
+    k64, v64, q64 = k.astype(np.float64), v.astype(np.float64), q.astype(np.float64)
+    P = Dg * Shat
+    X = P + float(beta) * np.outer(k64, v64 - k64 @ P)          # Eq. delta_update, in fp64
+    yref = X.T @ q64
+    assert np.abs(y - yref).max() <= 2e-6 * np.abs(yref).max()
+    # the new page is the fit of the fp32 tile X
+    page_ref = oracle.encode_head(X.astype(np.float32), unit, rb, w)
+    z1 = oracle.unpack_head(page1, unit, rb)[2]
+    z2 = oracle.unpack_head(page_ref, unit, rb)[2]
+    assert np.mean(z1 != z2) <= 1e-3
+
+
+def test_error_propagation_prop1(oracle, rng):
+    """E_t = A_t E_{t-1} + eps_t;  y_hat_t - y_t = (A_t E_{t-1})^T q_t."""
+    S = (rng.standard_normal((D, D))).astype(np.float32)
+    rb = np.full(D, 4, np.int8)
+    w = np.ones(D, np.float32)
+    page = oracle.encode_head(S, HEAD, rb, w)
+    Sref = S.copy()
+    for _ in range(5):
+        q, k, v, beta, gate = _inp(rng, False)
+        E = oracle.decode_head(page, HEAD, rb) - Sref.astype(np.float64)
+        page, yq = oracle.step_head(page, HEAD, rb, w, q, k, v, beta, gate)
+        Sref, yr = oracle.delta_step(Sref, q, k, v, beta, gate)
+        A = (np.eye(D) - float(beta) * np.outer(k, k).astype(np.float64)) * float(gate[0])
+        pred = (A @ E).T @ q.astype(np.float64)
+        assert np.abs((yq.astype(np.float64) - yr) - pred).max() <= 1e-4 * np.abs(yr).max()
+
+
+def test_calibration_omega_and_logret(oracle):
+    wl = W.WORKLOADS["gqa"].replace(batch=3)
+    mp = W.model_params(wl)
+    inp = W.step_inputs(wl, mp, W.STREAM_CALIB, 0, 0, batch=3)
+    om = np.zeros((wl.hv, D))
+    lr = np.zeros(wl.hv)
+    oracle.calib_observe(inp, om, lr)
+    for h in (0, 5, 31):
+        ref = np.zeros(D)
+        for b in range(3):
+            g = oracle.row_impact(inp.q[b, h // 2], inp.k[b, h // 2], inp.beta[b, h],
+                                  inp.gate[b, h], dense=True)
+            ref += g * g
+        assert np.allclose(om[h], ref, rtol=1e-10)
+        assert np.isclose(lr[h], np.sum(np.log(inp.gate[:, h].astype(np.float64))))
+
+
+def test_calibration_distortion_driver(oracle, rng):
+    S = (rng.standard_normal((2, 3, D, D))).astype(np.float32)
+    w = np.exp(rng.normal(0, 0.3, (3, D))).astype(np.float32)
+    acc = np.zeros((3, 4))
+    oracle.calib_distortion(HEAD, S, w, (4, 6, 8), None, 1, acc)
+    for h in range(3):
+        for kk, b in enumerate((4, 6, 8)):
+            rb = np.full(D, b, np.int8)
+            ref = 0.0
+            for s in range(2):
+                R = oracle.decode_head(oracle.encode_head(S[s, h], HEAD, rb, w[h]), HEAD, rb)
+                ref += np.sum(w[h][:, None].astype(np.float64) ** 2 * (R - S[s, h]) ** 2) / D / D
+            assert np.isclose(acc[h, kk], ref, rtol=1e-12)
+        assert acc[h, 0] > acc[h, 1] > acc[h, 2] > acc[h, 3] >= 0
+
+
+def test_end_to_end_tiny_calibration_and_plan(oracle):
+    wl = W.WORKLOADS["tiny"]
+    st = oracle.calibrate(wl, seqs=2, steps=32)
+    plan = oracle.plan_from_stats(wl, st)
+    assert plan.unit_bits.shape == (4,)
+    assert np.sum(plan.unit_bits) <= 6 * 4
+    assert plan.slot_stride == int(np.sum(plan.head_bytes))
