@@ -1,0 +1,354 @@
+"""Timing of the STEPQuant decode step on the 1024-slot serving pool.
+
+One step = one decode token through all 16 recurrent layers for the 1024 active
+slots (16 launches of the fused kernel, one per layer), i.e. 524,288 head-state
+updates. Prints one JSON line (see the keys below). `--impl reference` times
+the CPU oracle on a bounded sample of the same workload instead.
+
+Multi-GPU: every (slot, layer, head) update is independent and the path has no
+exchange step, so N ranks run N independent replicas of the workload (weak
+scaling, no collective on the data path); the value sums all ranks' updates
+over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "head-state decode updates/sec and achieved HBM GB/s (fraction of peak) at 1 GB300"
+UNIT = "head-updates/s"
+WORKLOAD = "pool"
+
+
+def _peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return {}
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self._stop = threading.Event()
+        self._t = None
+
+    def start(self):
+        def run():
+            while not self._stop.is_set():
+                try:
+                    out = subprocess.run(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits"], capture_output=True,
+                                         text=True, timeout=5).stdout.strip()
+                    if out:
+                        self.rows.append([x.strip() for x in out.split(",")])
+                except Exception:
+                    pass
+                self._stop.wait(0.2)
+        self._t = threading.Thread(target=run, daemon=True)
+        self._t.start()
+
+    def stop(self):
+        self._stop.set()
+        if self._t:
+            self._t.join(timeout=10)
+        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in self.rows for k in range(4)
+                          if len(r) > 3 + k and r[3 + k].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(self.rows)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def cpu_baseline(wl, units: int, min_seconds: float = 10.0):
+    """The oracle as it stands, on a bounded sample of the workload (all host cores):
+    decode steps of one layer for units / 32 slots, repeated until `min_seconds`."""
+    import oracle as O
+    from paper_2609_38169_gb300 import workloads as W
+    wl1 = wl.replace(layers=1)
+    st = O.calibrate(wl1, seqs=2, steps=16)
+    oplan = O.plan_from_stats(wl1, st)
+    mp = W.model_params(wl)
+    B = max(1, units // wl.hv)
+    slots = np.arange(B, dtype=np.int32)
+    S = W.random_states(wl, B * wl.hv).reshape(B, wl.hv, 128, 128)
+    pool = np.zeros(B * oplan.slot_stride, np.uint8)
+    O.pool_encode(oplan, pool, 0, slots, S)
+    del S
+    done, elapsed, step = 0, 0.0, 0
+    while elapsed < min_seconds or step == 0:
+        inp = W.step_inputs(wl, mp, W.STREAM_DECODE, step, 0, batch=B)
+        t0 = time.perf_counter()
+        O.pool_step(oplan, pool, 0, slots, inp)
+        elapsed += time.perf_counter() - t0
+        done += B * wl.hv
+        step += 1
+    return {"value": done / elapsed, "unit": UNIT, "cores": O.num_threads(), "kind": "oracle",
+            "sample": f"{step} decode steps of one layer for {B} slots x {wl.hv} heads "
+                      f"({done} head updates) of the {wl.name} workload, {elapsed:.1f} s"}
+
+
+def run_reference(args):
+    """The CPU oracle timed as the reference arm (rank 0 only)."""
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return
+    from paper_2609_38169_gb300 import workloads as W
+    wl = W.WORKLOADS[WORKLOAD]
+    per_step_units = args.ref_units
+    vals = []
+    for _ in range(args.warmup):
+        cpu_baseline(wl, per_step_units, min_seconds=0.0)
+    for _ in range(args.steps):
+        vals.append(cpu_baseline(wl, per_step_units, min_seconds=0.0))
+    v = statistics.median(x["value"] for x in vals)
+    ms = 1e3 * per_step_units / v
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": "serving state pool: 16 layers x 32 heads, 1024 slots, d=128, "
+                                   "nominal 6-bit STEPQuant (oracle on a bounded sample)",
+                       "sample_units_per_step": per_step_units},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": vals[-1]["cores"], "kind": "oracle",
+                             "sample": vals[-1]["sample"]},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="stepq", choices=["stepq", "reference"])
+    ap.add_argument("--no-baselines", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-units", type=int, default=4096)
+    ap.add_argument("--ref-units", type=int, default=1024)
+    ap.add_argument("--calib-steps", type=int, default=256)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import paper_2609_38169_gb300 as P
+    from paper_2609_38169_gb300 import workloads as W
+
+    world, rank, local = dist_setup()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    wl = W.WORKLOADS[WORKLOAD]
+    cfg = P.Config.from_workload(wl)
+    L, Hv, Hk, B = wl.layers, wl.hv, wl.hk, wl.batch
+
+    # ---- offline: calibration and plan (not timed) ----
+    st = P.calibrate(cfg, wl, device=dev, steps=args.calib_steps, device_inputs=True)
+    plan = P.stepq_fit_scales(cfg, st.omega, st.mean_log_ret, st.dist, st.pivot)
+    mp_dev = W.model_params_torch(W.model_params(wl), dev)
+
+    # ---- initial states: 32 FP32 warm-up steps from zero, then pack ----
+    fp32_pool = torch.zeros((wl.pool_slots, L, Hv, 128, 128), dtype=torch.float32, device=dev)
+    all_slots = torch.arange(wl.pool_slots, dtype=torch.int32, device=dev)
+    y_tmp = torch.empty((wl.pool_slots, Hv, 128), dtype=torch.float32, device=dev)
+    for t in range(wl.warmup_steps):
+        for layer in range(L):
+            q, k, v, beta, gate = W.torch_step_inputs(wl, mp_dev, t, layer, dev, W.STREAM_WARMUP,
+                                                      batch=wl.pool_slots)
+            P.stepq_fp32_decode_step(cfg, layer, fp32_pool, all_slots, q, k, v, beta, gate, y_tmp)
+    pool = P.alloc_pool(plan, wl.pool_slots, dev)
+    P.stepq_quantize_pool(plan, -1, fp32_pool, all_slots, pool)
+    int8_stride = P.stepq_intb_slot_bytes(cfg, 8)
+    int8_pool = None
+    if not args.no_baselines:
+        int8_pool = torch.zeros(wl.pool_slots * int8_stride, dtype=torch.uint8, device=dev)
+        P.stepq_intb_quantize_pool(cfg, 8, -1, fp32_pool, all_slots, int8_pool)
+    else:
+        del fp32_pool
+        fp32_pool = None
+    torch.cuda.synchronize()
+    assert P.stepq_device_error() == 0
+
+    slots = torch.from_numpy(W.slot_permutation(wl)).to(dev)
+    n_inputs = 2                       # distinct token steps of inputs, cycled
+    inputs = [[W.torch_step_inputs(wl, mp_dev, 1000 + s, layer, dev) for layer in range(L)]
+              for s in range(n_inputs)]
+    y = torch.empty((L, B, Hv, 128), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step_stepq(s, ev=None):
+        for layer in range(L):
+            q, k, v, beta, gate = inputs[s % n_inputs][layer]
+            if ev is not None:
+                ev[layer][0].record(stream)
+            P.stepq_decode_step(plan, layer, pool, slots, q, k, v, beta, gate, y[layer],
+                                pool_slots=wl.pool_slots)
+            if ev is not None:
+                ev[layer][1].record(stream)
+
+    def step_fp32(s):
+        for layer in range(L):
+            q, k, v, beta, gate = inputs[s % n_inputs][layer]
+            P.stepq_fp32_decode_step(cfg, layer, fp32_pool, slots, q, k, v, beta, gate, y[layer],
+                                     pool_slots=wl.pool_slots)
+
+    def step_int8(s):
+        for layer in range(L):
+            q, k, v, beta, gate = inputs[s % n_inputs][layer]
+            P.stepq_intb_decode_step(cfg, 8, layer, int8_pool, slots, q, k, v, beta, gate, y[layer],
+                                     pool_slots=wl.pool_slots)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    def timed(fn, steps, warmup, per_launch=False):
+        for s in range(warmup):
+            fn(s)
+        evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for _ in range(L)] for _ in range(steps)] if per_launch else None
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for s in range(steps):
+            if per_launch:
+                fn(s, evs[s])
+            else:
+                fn(s)
+        e1.record(stream)
+        barrier()
+        total_ms = e0.elapsed_time(e1)
+        launch_ms = None
+        if per_launch:
+            launch_ms = [a.elapsed_time(b) for row in evs for (a, b) in row]
+        return total_ms, launch_ms
+
+    clocks = ClockSampler(dev.index if dev.index is not None else 0)
+    clocks.start()
+    total_ms, launch_ms = timed(step_stepq, args.steps, args.warmup, per_launch=True)
+    clk = clocks.stop()
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    assert P.stepq_device_error() == 0
+    units_per_step = L * B * Hv
+    value = world * units_per_step * args.steps / (total_ms / 1e3)
+
+    # algorithmic bytes per launch: each head page read and written once, plus
+    # q, k (per key head), v, beta, gate read and y written
+    head_bytes = plan.head_bytes.reshape(L, Hv).astype(np.int64)
+    gate_b = 4 * (128 if cfg.unit_rows else 1)
+    io_b = B * (Hk * 2 * 512 + Hv * (512 + 4 + gate_b + 512))
+    layer_bytes = [int(B * 2 * head_bytes[l].sum() + io_b) for l in range(L)]
+    avg_launch_s = statistics.mean(launch_ms) / 1e3
+    achieved = statistics.mean(layer_bytes) / avg_launch_s / 1e9
+    peaks = _peaks()
+    peak = peaks.get("hbm_gbs", 6800.0)
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": None,
+                "peak_source": "measured" if "hbm_gbs" in peaks else "fallback",
+                "bytes_per_launch": statistics.mean(layer_bytes),
+                "avg_launch_us": avg_launch_s * 1e6}
+
+    # ---- end to end through the public API with host buffers ----
+    h_in = []
+    for layer in range(L):
+        h_in.append([x.cpu().pin_memory() for x in inputs[0][layer]])
+    d_in = [[torch.empty_like(x) for x in inputs[0][layer]] for layer in range(L)]
+    h_y = torch.empty((L, B, Hv, 128), dtype=torch.float32).pin_memory()
+    h2d = sum(x.numel() * x.element_size() for row in h_in for x in row)
+    d2h = h_y.numel() * 4
+
+    def step_e2e(s):
+        for layer in range(L):
+            for dst, src in zip(d_in[layer], h_in[layer]):
+                dst.copy_(src, non_blocking=True)
+            q, k, v, beta, gate = d_in[layer]
+            P.stepq_decode_step(plan, layer, pool, slots, q, k, v, beta, gate, y[layer],
+                                pool_slots=wl.pool_slots)
+        h_y.copy_(y, non_blocking=True)
+
+    e2e_ms, _ = timed(step_e2e, max(3, args.steps // 2), 2)
+    e2e_steps = max(3, args.steps // 2)
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e = {"value": world * units_per_step * e2e_steps / (e2e_ms / 1e3), "unit": UNIT,
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    baselines = {}
+    if not args.no_baselines:
+        nb = max(3, args.steps // 2)
+        fp_ms, _ = timed(step_fp32, nb, 2)
+        i8_ms, _ = timed(step_int8, nb, 2)
+        fp_bytes = B * Hv * (2 * 65536) + io_b
+        i8_bytes = B * Hv * 2 * (256 + 16384) + io_b
+        baselines = {
+            "fp32_state": {"value": units_per_step * nb / (fp_ms / 1e3), "unit": UNIT,
+                           "ms_per_step": fp_ms / nb,
+                           "achieved_gbs": L * fp_bytes * nb / (fp_ms / 1e3) / 1e9},
+            "int8_rowwise": {"value": units_per_step * nb / (i8_ms / 1e3), "unit": UNIT,
+                             "ms_per_step": i8_ms / nb,
+                             "achieved_gbs": L * i8_bytes * nb / (i8_ms / 1e3) / 1e9},
+        }
+
+    if rank == 0:
+        cpu = None
+        if not args.no_cpu_baseline and world == 1:
+            cpu = cpu_baseline(wl, args.cpu_units)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "serving state pool: 16 Delta-rule layers x 32 heads, d_k=d_v=128, "
+                                   "1024 request slots (random permutation), nominal 6-bit STEPQuant, "
+                                   "one step = one token through all 16 layers",
+                       "layers": L, "heads": Hv, "slots": B, "pool_bytes": plan.slot_stride * wl.pool_slots,
+                       "slot_stride": plan.slot_stride, "l2": "inputs larger than L2 (pool 6.5 GB)",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": L * args.steps, "clocks": clk, "baselines": baselines,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

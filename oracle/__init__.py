@@ -104,11 +104,18 @@ def _declare(L):
         fn.argtypes = args
 
 
+class _Ptr(C.c_void_p):
+    """A pointer argument that keeps its numpy array alive until the call returns."""
+    __slots__ = ("_keep",)
+
+
 def _p(a: np.ndarray | None):
     if a is None:
         return None
     assert a.flags["C_CONTIGUOUS"], "oracle arrays must be C-contiguous"
-    return a.ctypes.data
+    ptr = _Ptr(a.ctypes.data)
+    ptr._keep = a
+    return ptr
 
 
 def _f32(a):

@@ -1,0 +1,59 @@
+// Sticky device error word and the slot-list validator.
+//
+// Kernels never trap: a unit whose slot id is out of range is skipped and the
+// first such status is latched in a per-device word that stepq_device_error()
+// reads and clears.
+#include "device.cuh"
+#include "internal.h"
+
+namespace stepq {
+
+__device__ unsigned int g_error_word;
+
+unsigned int *device_error_word() {
+    static unsigned int *addr[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    if (!addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+        addr[dev] = (unsigned int *)p;
+    }
+    return addr[dev];
+}
+
+stepq_status read_device_error(cudaStream_t s) {
+    unsigned int *w = device_error_word();
+    if (!w) return STEPQ_ERR_CUDA;
+    unsigned int v = 0;
+    if (cudaMemcpyAsync(&v, w, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaMemsetAsync(w, 0, sizeof(v), s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess)
+        return STEPQ_ERR_CUDA;
+    return (stepq_status)v;
+}
+
+// Marks each slot in a bitmap with atomicOr; a bit already set means a repeat.
+__global__ void validate_slots_kernel(const int32_t *slots, int B, int pool_slots,
+                                      uint32_t *bitmap, int32_t *status) {
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= B) return;
+    const int s = slots[t];
+    if (s < 0 || s >= pool_slots) {
+        atomicCAS((unsigned int *)status, 0u, (unsigned int)STEPQ_ERR_SLOT_RANGE);
+        return;
+    }
+    const uint32_t bit = 1u << (s & 31);
+    if (atomicOr(&bitmap[s >> 5], bit) & bit)
+        atomicCAS((unsigned int *)status, 0u, (unsigned int)STEPQ_ERR_DUP_SLOT);
+}
+
+stepq_status launch_validate_slots(const int32_t *slots, int B, int pool_slots,
+                                   uint32_t *scratch, int32_t *status, cudaStream_t s) {
+    if (cudaMemsetAsync(scratch, 0, ((size_t)pool_slots + 31) / 32 * 4, s) != cudaSuccess ||
+        cudaMemsetAsync(status, 0, sizeof(int32_t), s) != cudaSuccess)
+        return STEPQ_ERR_CUDA;
+    if (B > 0) validate_slots_kernel<<<(B + 255) / 256, 256, 0, s>>>(slots, B, pool_slots, scratch, status);
+    return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;
+}
+
+}  // namespace stepq

@@ -176,7 +176,8 @@ def random_states(wl: Workload, n: int, seed: int = 5, scale: float = 1.0) -> np
 
 # ---- device-side draws for full-size timing runs (torch Philox; same recipe) ----
 
-def torch_step_inputs(wl: Workload, mp_dev: dict, step: int, layer: int, device, stream: int = STREAM_DECODE):
+def torch_step_inputs(wl: Workload, mp_dev: dict, step: int, layer: int, device,
+                      stream: int = STREAM_DECODE, batch: int | None = None):
     """Same distributions as `step_inputs`, drawn on the GPU with torch's generator.
 
     Used where the oracle never sees the values (timing runs). `mp_dev` holds the
@@ -186,7 +187,7 @@ def torch_step_inputs(wl: Workload, mp_dev: dict, step: int, layer: int, device,
     import torch
     g = torch.Generator(device=device)
     g.manual_seed((wl.seed * 1_000_003 + stream * 10_007 + step * 131 + layer) & 0x7FFF_FFFF_FFFF)
-    b = wl.batch
+    b = wl.batch if batch is None else batch
     f = torch.float32
     q = torch.randn((b, wl.hk, DK), generator=g, device=device, dtype=f)
     n = torch.randn((b, wl.hk, DK), generator=g, device=device, dtype=f) * mp_dev["k_scale"][layer][None]
