@@ -152,6 +152,8 @@ def main():
     ap.add_argument("--cpu-units", type=int, default=4096)
     ap.add_argument("--ref-units", type=int, default=1024)
     ap.add_argument("--calib-steps", type=int, default=256)
+    ap.add_argument("--slots", type=int, default=None, help="smaller pool (profiling cases only)")
+    ap.add_argument("--layers", type=int, default=None, help="fewer layers (profiling cases only)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -168,6 +170,9 @@ def main():
     dev = torch.device("cuda", local if world > 1 else 0)
     torch.cuda.set_device(dev)
     wl = W.WORKLOADS[WORKLOAD]
+    if args.slots or args.layers:
+        wl = wl.replace(batch=args.slots or wl.batch, pool_slots=args.slots or wl.pool_slots,
+                        layers=args.layers or wl.layers)
     cfg = P.Config.from_workload(wl)
     L, Hv, Hk, B = wl.layers, wl.hv, wl.hk, wl.batch
 
@@ -233,13 +238,14 @@ def main():
             dist.barrier()
         torch.cuda.synchronize(dev)
 
-    def timed(fn, steps, warmup, per_launch=False):
+    def timed(fn, steps, warmup, per_launch=False, name="timed"):
         for s in range(warmup):
             fn(s)
         evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 for _ in range(L)] for _ in range(steps)] if per_launch else None
         barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.nvtx.range_push(name)
         e0.record(stream)
         for s in range(steps):
             if per_launch:
@@ -247,6 +253,7 @@ def main():
             else:
                 fn(s)
         e1.record(stream)
+        torch.cuda.nvtx.range_pop()
         barrier()
         total_ms = e0.elapsed_time(e1)
         launch_ms = None
@@ -256,7 +263,7 @@ def main():
 
     clocks = ClockSampler(dev.index if dev.index is not None else 0)
     clocks.start()
-    total_ms, launch_ms = timed(step_stepq, args.steps, args.warmup, per_launch=True)
+    total_ms, launch_ms = timed(step_stepq, args.steps, args.warmup, per_launch=True, name="stepq_decode")
     clk = clocks.stop()
     if world > 1:
         import torch.distributed as dist
@@ -301,7 +308,7 @@ def main():
                                 pool_slots=wl.pool_slots)
         h_y.copy_(y, non_blocking=True)
 
-    e2e_ms, _ = timed(step_e2e, max(3, args.steps // 2), 2)
+    e2e_ms, _ = timed(step_e2e, max(3, args.steps // 2), 2, name="stepq_e2e")
     e2e_steps = max(3, args.steps // 2)
     if world > 1:
         import torch.distributed as dist
@@ -314,8 +321,8 @@ def main():
     baselines = {}
     if not args.no_baselines:
         nb = max(3, args.steps // 2)
-        fp_ms, _ = timed(step_fp32, nb, 2)
-        i8_ms, _ = timed(step_int8, nb, 2)
+        fp_ms, _ = timed(step_fp32, nb, 2, name="fp32_decode")
+        i8_ms, _ = timed(step_int8, nb, 2, name="int8_decode")
         fp_bytes = B * Hv * (2 * 65536) + io_b
         i8_bytes = B * Hv * 2 * (256 + 16384) + io_b
         baselines = {
@@ -335,11 +342,11 @@ def main():
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": "serving state pool: 16 Delta-rule layers x 32 heads, d_k=d_v=128, "
-                                   "1024 request slots (random permutation), nominal 6-bit STEPQuant, "
-                                   "one step = one token through all 16 layers",
+            "config": {"workload": f"serving state pool: {L} Delta-rule layers x {Hv} heads, d_k=d_v=128, "
+                                   f"{B} request slots (random permutation), nominal 6-bit STEPQuant, "
+                                   f"one step = one token through all {L} layers",
                        "layers": L, "heads": Hv, "slots": B, "pool_bytes": plan.slot_stride * wl.pool_slots,
-                       "slot_stride": plan.slot_stride, "l2": "inputs larger than L2 (pool 6.5 GB)",
+                       "slot_stride": plan.slot_stride, "l2": f"inputs larger than L2 (pool {plan.slot_stride * wl.pool_slots / 1e9:.2f} GB)",
                        "parallelism": f"replicas x{world}"},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": L * args.steps, "clocks": clk, "baselines": baselines,
