@@ -12,7 +12,8 @@
  *  - r_i = fp16(clamp(sqrt(m_i) * w_i^(-1/2), 2^-14, 65504)), the FP16 clamp of
  *    the baseline's scale storage (App. B.5);
  *  - the column fit starts from the clip-free value
- *    c0_j = max_{i in I} |X_ij| / (r_i zs_i qmax_i), then applies `fit_iters`
+ *    c0_j = max_{i in I} |X_ij| / (r_i zs_i qmax_i) (evaluated in fp32 as
+ *    max_i fp32(fp32(|X_ij| rho_i) / qmax_i)), then applies `fit_iters`
  *    fixed-code updates c_j = sum w_i^2 v_ij X_ij / sum w_i^2 v_ij^2 (App. C.1),
  *    a zero denominator keeping the current iterate, floor 2^-14, cap 65504;
  *  - "round to the nearest level" is round-half-to-even of the fp32 value
@@ -21,10 +22,14 @@
  *  - codes are stored offset-binary u = q + 2^(b-1), LSB-first per row.
  *
  * Page layout of one head (all pieces 16-byte multiples):
- *   integer head unit: r[128] fp16 | c[128] fp16 | 128 rows x 16b bytes
- *   pivot head unit:   128 rows x 256 bytes (fp16 values)
- *   row-unit head:     r[128] fp16 | c[128] fp16 | row i: 16 b_i bytes
- *                      (b_i = 16 marks an FP16 pivot row, 256 bytes)
+ *   integer head unit: r[128] fp16 | c[128] fp16 | codes in band-major order:
+ *                      for band w = 0..7 (rows 16w..16w+15), for column j,
+ *                      the 16 codes of rows 16w.. in that column (2b bytes)
+ *   pivot head unit:   the same band-major order of fp16 values (32 bytes
+ *                      per band column), no scales
+ *   row-unit head:     r[128] fp16 | c[128] fp16 | row i: 16 b_i bytes with the
+ *                      codes of columns 0..127 (b_i = 16 marks an FP16 pivot
+ *                      row, 256 bytes)
  */
 #include <math.h>
 #include <stdlib.h>
@@ -59,13 +64,20 @@ size_t or_head_bytes(int unit_kind, const int8_t *rb)
     return n;
 }
 
-static size_t row_offset(int unit_kind, const int8_t *rb, int i)
+/* Byte offset of the stream holding element (i, j) and its bit position in it. */
+static size_t elem_stream(int unit_kind, const int8_t *rb, int i, int j, int *bitpos)
 {
-    if (is_pivot_head(unit_kind, rb))
-        return (size_t)i * 256;
+    int b = rb[i];
+    if (unit_kind == OR_UNIT_HEAD) {
+        size_t base = is_pivot_head(unit_kind, rb) ? 0 : 512;
+        size_t chunk = (size_t)(i / 16) * OR_D + (size_t)j;        /* band-major chunks */
+        *bitpos = (i % 16) * b;
+        return base + chunk * 2 * (size_t)b;
+    }
     size_t off = 512;
     for (int t = 0; t < i; t++)
         off += 16 * (size_t)rb[t];
+    *bitpos = j * b;
     return off;
 }
 
@@ -105,14 +117,15 @@ void or_unpack_head(const uint8_t *page, int unit_kind, const int8_t *rb,
         c[i] = ph ? 0 : get_u16(page + 256 + 2 * i);
     }
     for (int i = 0; i < OR_D; i++) {
-        const uint8_t *row = page + row_offset(unit_kind, rb, i);
         int b = rb[i];
         for (int j = 0; j < OR_D; j++) {
+            int pos;
+            const uint8_t *stream = page + elem_stream(unit_kind, rb, i, j, &pos);
             if (b == OR_PIVOT_BITS) {
-                piv[i * OR_D + j] = get_u16(row + 2 * j);
+                piv[i * OR_D + j] = get_u16(stream + pos / 8);
                 codes[i * OR_D + j] = 0;
             } else {
-                unsigned u = get_bits(row, j * b, b);
+                unsigned u = get_bits(stream, pos, b);
                 codes[i * OR_D + j] = (int8_t)((int)u - (1 << (b - 1)));
                 piv[i * OR_D + j] = 0;
             }
@@ -158,14 +171,14 @@ void or_decode_head_f32(const uint8_t *page, int unit_kind, const int8_t *rb, fl
 static void fit_head(const float *X, int unit_kind, const int8_t *rb, const float *w,
                      int fit_iters, double *r, float *rho, float *c, int8_t *z_last)
 {
-    float rho_max[OR_D];      /* fp32(1 / (r_i zs_i qmax_i)) */
+    float mu[OR_D];           /* fp32(1 / qmax_i) */
     int in_fit[OR_D];         /* non-pivot integer rows: the set I */
     for (int i = 0; i < OR_D; i++) {
         int b = rb[i];
         in_fit[i] = (b != OR_PIVOT_BITS);
         if (!in_fit[i]) {
             r[i] = 0.0;
-            rho[i] = rho_max[i] = 0.0f;
+            rho[i] = mu[i] = 0.0f;
             continue;
         }
         /* Row factors: m_i = (1/d_v) sum_j |X_ij|, r_i = m_i^(1/2) w_i^(-1/2). */
@@ -178,15 +191,17 @@ static void fit_head(const float *X, int unit_kind, const int8_t *rb, const floa
         r[i] = or_fp16_round(clampd(t, F16_MIN_NORMAL, F16_MAX));
         double zs = zs_of(unit_kind, b);
         rho[i] = (float)(1.0 / (r[i] * zs));
-        rho_max[i] = (float)(1.0 / (r[i] * zs * qmax_of(b)));
+        mu[i] = (float)(1.0 / qmax_of(b));
     }
-    /* Column factors: clip-free start, then fixed-code least-squares updates of
-     * min_c sum_ij w_i^2 (X_ij - r_i c_j z_ij)^2 over the rows in I. */
+    /* Column factors: clip-free start c0_j = max_i |X_ij| / (r_i zs_i qmax_i),
+     * evaluated as max_i fp32(fp32(|X_ij| rho_i) mu_i), then fixed-code
+     * least-squares updates of min_c sum_ij w_i^2 (X_ij - r_i c_j z_ij)^2 over
+     * the rows in I. */
     for (int j = 0; j < OR_D; j++) {
         float cmax = 0.0f;
         for (int i = 0; i < OR_D; i++)
             if (in_fit[i]) {
-                float a = mul32(fabsf(X[i * OR_D + j]), rho_max[i]);
+                float a = mul32(mul32(fabsf(X[i * OR_D + j]), rho[i]), mu[i]);
                 if (a > cmax)
                     cmax = a;
             }
@@ -231,9 +246,11 @@ void or_encode_head(const float *X, int unit_kind, const int8_t *rb, const float
 {
     if (is_pivot_head(unit_kind, rb)) {             /* FP16 pivot head */
         for (int i = 0; i < OR_D; i++)
-            for (int j = 0; j < OR_D; j++)
-                put_u16(page + (size_t)i * 256 + 2 * j,
-                        or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
+            for (int j = 0; j < OR_D; j++) {
+                int pos;
+                uint8_t *stream = page + elem_stream(unit_kind, rb, i, j, &pos);
+                put_u16(stream + pos / 8, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
+            }
         return;
     }
     double r[OR_D];
@@ -251,18 +268,18 @@ void or_encode_head(const float *X, int unit_kind, const int8_t *rb, const float
         put_u16(page + 256 + 2 * i, or_fp16_encode(c16[i]));
     }
     for (int i = 0; i < OR_D; i++) {
-        uint8_t *row = page + row_offset(unit_kind, rb, i);
         int b = rb[i];
-        if (b == OR_PIVOT_BITS) {
-            for (int j = 0; j < OR_D; j++)
-                put_u16(row + 2 * j, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
-            continue;
-        }
-        int qm = qmax_of(b);
+        int qm = b == OR_PIVOT_BITS ? 0 : qmax_of(b);
         for (int j = 0; j < OR_D; j++) {
+            int pos;
+            uint8_t *stream = page + elem_stream(unit_kind, rb, i, j, &pos);
+            if (b == OR_PIVOT_BITS) {
+                put_u16(stream + pos / 8, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
+                continue;
+            }
             float t = mul32(mul32(X[i * OR_D + j], rho[i]), gamma[j]);
             int qv = (int)clampd(rint((double)t), -qm, qm);
-            put_bits(row, j * b, b, (unsigned)(qv + (1 << (b - 1))));
+            put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1))));
         }
     }
 }

@@ -212,6 +212,7 @@ extern "C" const char *stepq_status_str(stepq_status s) {
     case STEPQ_ERR_CUDA: return "CUDA runtime error";
     case STEPQ_ERR_BUDGET: return "bit budget cannot be met by the candidates";
     case STEPQ_ERR_UNSUPPORTED: return "unsupported configuration";
+    case STEPQ_ERR_TIMEOUT: return "a device-side wait exceeded its bound";
     }
     return "unknown status";
 }

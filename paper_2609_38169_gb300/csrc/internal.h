@@ -87,6 +87,17 @@ stepq_status launch_quantize(const stepq_plan *p, int layer, const float *states
 stepq_status launch_dequantize(const stepq_plan *p, int layer, const uint8_t *pool, int pool_slots,
                                const int32_t *slots, int B, float *states, size_t state_stride_b,
                                cudaStream_t s);
+// heads.cu (head units, band-major pages)
+stepq_status launch_decode_heads(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
+                                 const int32_t *slots, int B, const float *q, const float *k,
+                                 const float *v, const float *beta, const float *gate, float *y,
+                                 cudaStream_t s);
+stepq_status launch_quantize_heads(const stepq_plan *p, int layer, const float *states,
+                                   size_t stride_b, const int32_t *slots, int B, uint8_t *pool,
+                                   int pool_slots, cudaStream_t s);
+stepq_status launch_dequantize_heads(const stepq_plan *p, int layer, const uint8_t *pool,
+                                     int pool_slots, const int32_t *slots, int B, float *states,
+                                     size_t stride_b, cudaStream_t s);
 // baselines.cu
 stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool, int pool_slots,
                                 const int32_t *slots, int B, const float *q, const float *k,

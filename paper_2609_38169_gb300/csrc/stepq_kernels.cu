@@ -1,4 +1,5 @@
-// The fused STEPQuant decode step and the pool pack/unpack kernels (sm_103a).
+// Row-unit (KDA) decode step, pool pack/unpack and the calibration distortion
+// kernel (sm_103a). Head units (GDN) run the pipelined kernels of heads.cu.
 //
 // One 256-thread CTA owns one (slot, value head) page: it stages the packed
 // head segment in shared memory with 128-bit loads, reconstructs the tile into
@@ -11,7 +12,8 @@
 // the tile X is fp32; r_i = fp16(clamp(sqrt(m_i) * w_i^(-1/2), 2^-14, 65504));
 // rho_i = fp32(1/(r_i zs_i)); every code decision is rint(fp32(fp32(X rho_i)
 // gamma_j)) with gamma_j = fp32(1/c_j); c is fitted from the clip-free start
-// max_i |X_ij| rho_i / qmax_i by `fit_iters` fixed-code least-squares updates.
+// max_i fp32(fp32(|X_ij| rho_i) / qmax_i) by `fit_iters` fixed-code
+// least-squares updates.
 #include <cstdio>
 
 #include "device.cuh"
@@ -69,14 +71,14 @@ __device__ __forceinline__ void fit_scales(const Lane &L, const TileSmem &S, con
     float *colC = S.col;           // current column iterate
     float *colG = S.col + 128;     // its reciprocal
     float *colND = S.col + 256;    // [2][128] numerator / denominator
-    float rhom[4];
+    float mu[4];                   // fp32(1 / qmax_i)
     // Row factors r_i = m_i^(1/2) w_i^(-1/2).
 #pragma unroll
     for (int t = 0; t < 4; t++) {
         const int i = L.row(t);
         f.bits[t] = S.rbits[i];
         if (f.bits[t] == kPivot) {
-            f.rr[t] = f.rho[t] = rhom[t] = f.zsv[t] = 0.f;
+            f.rr[t] = f.rho[t] = mu[t] = f.zsv[t] = 0.f;
             f.qm[t] = 0;
             if (write_scales && L.cg == 0) page_r[i] = 0;
             continue;
@@ -89,10 +91,11 @@ __device__ __forceinline__ void fit_scales(const Lane &L, const TileSmem &S, con
         f.rr[t] = rf;
         f.zsv[t] = zs;
         f.rho[t] = __frcp_rn(rf * zs);
-        rhom[t] = __frcp_rn((rf * zs) * (float)f.qm[t]);
+        mu[t] = __frcp_rn((float)f.qm[t]);
         if (write_scales && L.cg == 0) page_r[i] = f16_bits(rf);
     }
-    // Clip-free column start: c0_j = max_i |X_ij| / (r_i zs_i qmax_i).
+    // Clip-free column start: c0_j = max_i |X_ij| / (r_i zs_i qmax_i), as
+    // max_i fp32(fp32(|X_ij| rho_i) mu_i).
     {
         float acc[1][16];
 #pragma unroll
@@ -101,7 +104,7 @@ __device__ __forceinline__ void fit_scales(const Lane &L, const TileSmem &S, con
         for (int t = 0; t < 4; t++)
 #pragma unroll
             for (int j = 0; j < 16; j++)
-                acc[0][j] = fmaxf(acc[0][j], __fmul_rn(fabsf(x[t][j]), rhom[t]));
+                acc[0][j] = fmaxf(acc[0][j], __fmul_rn(__fmul_rn(fabsf(x[t][j]), f.rho[t]), mu[t]));
         column_reduce<1, true>(L, acc, S.red, colC);
         if (L.tid < 128) {
             const float c = fminf(fmaxf(colC[L.tid], kF16Min), kF16Max);
@@ -519,6 +522,8 @@ stepq_status launch_decode(const stepq_plan *p, int layer, uint8_t *pool, int po
                            const int32_t *slots, int B, const float *q, const float *k,
                            const float *v, const float *beta, const float *gate, float *y,
                            cudaStream_t s) {
+    if (p->cfg.gate_kind == STEPQ_GATE_SCALAR)
+        return launch_decode_heads(p, layer, pool, pool_slots, slots, B, q, k, v, beta, gate, y, s);
     stepq_status st = prepare(p->device);
     if (st != STEPQ_OK) return st;
     DecodeArgs a{pool, p->slot_stride, pool_slots, slots, p->layer(layer), p->shape(),
@@ -530,6 +535,8 @@ stepq_status launch_decode(const stepq_plan *p, int layer, uint8_t *pool, int po
 stepq_status launch_quantize(const stepq_plan *p, int layer, const float *states,
                              size_t state_stride_b, const int32_t *slots, int B, uint8_t *pool,
                              int pool_slots, cudaStream_t s) {
+    if (p->cfg.gate_kind == STEPQ_GATE_SCALAR)
+        return launch_quantize_heads(p, layer, states, state_stride_b, slots, B, pool, pool_slots, s);
     stepq_status st = prepare(p->device);
     if (st != STEPQ_OK) return st;
     PoolArgs a{pool, p->slot_stride, pool_slots, slots, p->layer(layer), p->shape(),
@@ -541,6 +548,8 @@ stepq_status launch_quantize(const stepq_plan *p, int layer, const float *states
 stepq_status launch_dequantize(const stepq_plan *p, int layer, const uint8_t *pool, int pool_slots,
                                const int32_t *slots, int B, float *states, size_t state_stride_b,
                                cudaStream_t s) {
+    if (p->cfg.gate_kind == STEPQ_GATE_SCALAR)
+        return launch_dequantize_heads(p, layer, pool, pool_slots, slots, B, states, state_stride_b, s);
     stepq_status st = prepare(p->device);
     if (st != STEPQ_OK) return st;
     PoolArgs a{(uint8_t *)pool, p->slot_stride, pool_slots, slots, p->layer(layer), p->shape(),

@@ -86,14 +86,16 @@ def test_pivot_head_is_fp16(oracle, rng):
     rb = np.full(D, PIV, np.int8)
     page = oracle.encode_head(X, HEAD, rb, _w(rng))
     assert page.size == D * D * 2
-    vals = page.view(np.float16).reshape(D, D).astype(np.float64)
-    ref = np.float16(np.clip(X, -65504, 65504)).astype(np.float64)
-    assert np.array_equal(vals, ref)
+    # band-major: [band w][column j][row 16w + r]
+    vals = page.view(np.float16).reshape(8, D, 16).transpose(0, 2, 1).reshape(D, D)
+    ref = np.float16(np.clip(X, -65504, 65504))
+    assert np.array_equal(vals.astype(np.float64), ref.astype(np.float64))
 
 
 @pytest.mark.parametrize("b", [2, 4, 6, 8])
 def test_bit_layout_with_independent_unpacker(oracle, rng, b):
-    """Offset-binary codes u = q + 2^(b-1), LSB-first in each row's byte stream."""
+    """Head units: offset-binary codes u = q + 2^(b-1), LSB-first, in band-major
+    chunks (band w of 16 rows, column j: the 16 codes of rows 16w..16w+15)."""
     X = _state(rng)
     rb = np.full(D, b, np.int8)
     page = oracle.encode_head(X, HEAD, rb, _w(rng))
@@ -101,10 +103,32 @@ def test_bit_layout_with_independent_unpacker(oracle, rng, b):
     r16, c16, codes, _ = oracle.unpack_head(page, HEAD, rb)
     assert np.array_equal(page[:256].view(np.uint16), r16)
     assert np.array_equal(page[256:512].view(np.uint16), c16)
-    bits = np.unpackbits(page[512:].reshape(D, 16 * b), axis=1, bitorder="little")
-    u = (bits.reshape(D, D, b) * (1 << np.arange(b))).sum(-1)
+    bits = np.unpackbits(page[512:].reshape(8 * D, 2 * b), axis=1, bitorder="little")
+    u = (bits.reshape(8, D, 16, b) * (1 << np.arange(b))).sum(-1)     # [band][col][row in band]
+    u = u.transpose(0, 2, 1).reshape(D, D)
     assert np.array_equal(u - 2 ** (b - 1), codes.astype(np.int64))
     assert u.min() >= 1
+
+
+def test_row_unit_layout_with_independent_unpacker(oracle, rng):
+    """Row units: r | c | row i holds its 128 codes (b_i bits, LSB-first), FP16 rows
+    for pivots; rows follow each other in index order."""
+    X = _state(rng)
+    rb = _widths(rng, ROW)
+    page = oracle.encode_head(X, ROW, rb, _w(rng))
+    assert page.size == 512 + 16 * int(np.sum(rb.astype(np.int64)))
+    _, _, codes, piv = oracle.unpack_head(page, ROW, rb)
+    off = 512
+    for i in range(D):
+        b = int(rb[i])
+        row = page[off:off + 16 * b]
+        if b == PIV:
+            assert np.array_equal(row.view(np.uint16), piv[i])
+        else:
+            bits = np.unpackbits(row, bitorder="little").reshape(D, b)
+            u = (bits * (1 << np.arange(b))).sum(-1)
+            assert np.array_equal(u - 2 ** (b - 1), codes[i].astype(np.int64))
+        off += 16 * b
 
 
 def test_zero_state(oracle, rng):
