@@ -30,10 +30,11 @@ constexpr int kOffBars = 0;                            // uint64 [8]
 constexpr int kOffFlags = 64;                          // int [16]
 constexpr int kOffRed = 128;                           // float [2][8][128]
 constexpr int kOffCol = kOffRed + 2 * 8 * 128 * 4;     // float [4][128]
-constexpr int kOffRowC = kOffCol + 4 * 128 * 4;        // float4 [128]: a, kappa, beta*k, q
-constexpr int kOffRowF = kOffRowC + 128 * 16;          // float2 [128]: rho, alpha_ls
+constexpr int kOffRowC = kOffCol + 4 * 128 * 4;        // float4 [2][128]: kappa,kappa,bk',bk' | qa,qa,a,a
+constexpr int kOffRowF = kOffRowC + 256 * 16;          // float4 [128]: rho a, rho a, alpha_ls, alpha_ls
+constexpr int kOffRowA = kOffRowF + 128 * 16;          // float [128]: a_i
 constexpr int kMaxHv = 256;                            // value heads per layer (launch check)
-constexpr int kOffHead = kOffRowF + 128 * 8;           // u64 off[256] | u32 bytes[256] | u8 bits[256]
+constexpr int kOffHead = kOffRowA + 128 * 4;           // u64 off[256] | u32 bytes[256] | u8 bits[256]
 constexpr int kOffStages = (kOffHead + kMaxHv * 13 + 127) / 128 * 128;
 
 struct Smem {
@@ -41,7 +42,8 @@ struct Smem {
     int *flags;
     float *red, *colC, *colG, *colD, *colX;
     float4 *rowc;
-    float2 *rowf;
+    float4 *rowf;
+    float *rowa;
     uint64_t *hoff;
     uint32_t *hbytes;
     uint8_t *hbits;
@@ -55,7 +57,8 @@ struct Smem {
         colD = colC + 256;
         colX = colC + 384;
         rowc = (float4 *)(s + kOffRowC);
-        rowf = (float2 *)(s + kOffRowF);
+        rowf = (float4 *)(s + kOffRowF);
+        rowa = (float *)(s + kOffRowA);
         hoff = (uint64_t *)(s + kOffHead);
         hbytes = (uint32_t *)(s + kOffHead + kMaxHv * 8);
         hbits = s + kOffHead + kMaxHv * 12;
@@ -206,16 +209,17 @@ __device__ __forceinline__ void cols_to_red(const T &t, float *red, const float 
 
 // ---------------------------------------------------------------- the fit
 // Key-Row-Aware Dual-axis Fitting of the register tile (Sec. 4.3, App. C.1)
-// and packing into the page (App. C.3 step 6). x2 holds X (fp32) as column
-// pairs; rs[r] the partial |X| sums of the thread's rows over its 4 columns.
-// With y_part set, the readout partials ride on the same reduction round.
-// On return the page holds r, c and the codes. Requires the old page to be
-// fully consumed by every thread.
+// and packing into the page (App. C.3 step 6). The tile holds Z with
+// X_ij = a_i Z_ij (a_i > 0 a per-row factor: a_i = alpha r_i in the decode
+// step, 1 when packing a dense state); rs[r] holds the partial sums of |Z| of
+// the thread's rows over its 4 columns. Readout partials (y_part), when given,
+// ride on the column-start reduction round. On return the page holds r, c and
+// the codes. Requires the old page to be fully consumed by every thread.
 template <int B>
 __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *page, const float *w2v,
-                                         const float *wisv, uint64_t (&x2)[16][2], float (&rs)[16],
-                                         const float (&y_part)[4], bool with_y, float *y_out,
-                                         int fit_iters) {
+                                         const float *wisv, const float *a_row, uint64_t (&x2)[16][2],
+                                         float (&rs)[16], const float (&y_part)[4], bool with_y,
+                                         float *y_out, int fit_iters) {
     constexpr int qm = (1 << (B - 1)) - 1;
     constexpr float fqm = (float)qm;
     const float mu = __frcp_rn(fqm);
@@ -224,13 +228,16 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
     // Row factors r_i = m_i^(1/2) w_i^(-1/2), m_i = (1/128) sum_j |X_ij|.
     {
         int rr;
-        const float s = warp_row_sums(rs, t.l, rr);
+        const float sz = warp_row_sums(rs, t.l, rr);
         const int i = t.row(rr);
-        const float m = s * (1.0f / 128.0f);
+        const float a = a_row ? a_row[i] : 1.f;
+        const float m = (a * sz) * (1.0f / 128.0f);
         const float rf = __half2float(__float2half_rn(
             fminf(fmaxf(__fmul_rn(sqrtf(m), wisv[i]), kF16Min), kF16Max)));
         if ((t.l & 1) == 0) {
-            S.rowf[i] = make_float2(__frcp_rn(rf), w2v[i] * (rf * rf));
+            const float rho_a = __frcp_rn(rf) * a;                 // X' = rho_i X = (rho_i a_i) Z
+            const float al = w2v[i] * (rf * rf);                   // w_i^2 r_i^2
+            S.rowf[i] = make_float4(rho_a, rho_a, al, al);
             page_r[i] = f16_bits(rf);
         }
     }
@@ -239,7 +246,8 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
     float cm[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int r = 0; r < 16; r++) {
-        const uint64_t rho = f2s(S.rowf[t.row(r)].x);
+        const uint4 rf = *(const uint4 *)&S.rowf[t.row(r)];
+        const uint64_t rho = ((uint64_t)rf.y << 32) | rf.x;
         x2[r][0] = fmul2(x2[r][0], rho);
         x2[r][1] = fmul2(x2[r][1], rho);
         cm[0] = fmaxf(cm[0], fabsf(f2lo(x2[r][0])));
@@ -256,7 +264,10 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         }
         cols_to_red<2>(t, S.red, v);
     }
-    if (t.tid == 0) S.flags[1] = 0;
+    if (t.tid == 0) {
+        S.flags[1] = 0;
+        S.flags[2] = 0;
+    }
     __syncthreads();
     if (t.tid < 128) {
         float mx = S.red[t.tid];
@@ -267,6 +278,7 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         const float c = fminf(fmaxf(c0, kF16Min), kF16Max);
         S.colC[t.tid] = c;
         S.colG[t.tid] = __frcp_rn(c);
+        S.colX[t.tid] = mx;                               // max_i |X'_ij|
         if (with_y) {
             float s = S.red[8 * 128 + t.tid];
 #pragma unroll
@@ -282,10 +294,11 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         const bool clip = it > 0 || S.flags[1];
         const uint64_t g01 = f2(S.colG[t.col(0)], S.colG[t.col(1)]);
         const uint64_t g23 = f2(S.colG[t.col(2)], S.colG[t.col(3)]);
-        uint64_t n01 = 0, n23 = 0, d01 = 0, d23 = 0;
+        uint64_t n01 = 0, n23 = 0, d01 = 0, d23 = 0, e01 = 0, e23 = 0, h01 = 0, h23 = 0;
 #pragma unroll
         for (int r = 0; r < 16; r++) {
-            const uint64_t al = f2s(S.rowf[t.row(r)].y);
+            const uint4 rf = *(const uint4 *)&S.rowf[t.row(r)];
+            const uint64_t al = ((uint64_t)rf.w << 32) | rf.z;
             uint64_t q01 = fadd2(fadd2(fmul2(x2[r][0], g01), M2), nM2);
             uint64_t q23 = fadd2(fadd2(fmul2(x2[r][1], g23), M2), nM2);
             if (clip) {
@@ -293,11 +306,22 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
                 q23 = f2(fminf(fmaxf(f2lo(q23), -fqm), fqm), fminf(fmaxf(f2hi(q23), -fqm), fqm));
             }
             const uint64_t a01 = fmul2(al, q01), a23 = fmul2(al, q23);
-            n01 = ffma2(a01, x2[r][0], n01);
-            n23 = ffma2(a23, x2[r][1], n23);
-            d01 = ffma2(a01, q01, d01);
-            d23 = ffma2(a23, q23, d23);
+            if (r & 1) {
+                e01 = ffma2(a01, x2[r][0], e01);
+                e23 = ffma2(a23, x2[r][1], e23);
+                h01 = ffma2(a01, q01, h01);
+                h23 = ffma2(a23, q23, h23);
+            } else {
+                n01 = ffma2(a01, x2[r][0], n01);
+                n23 = ffma2(a23, x2[r][1], n23);
+                d01 = ffma2(a01, q01, d01);
+                d23 = ffma2(a23, q23, d23);
+            }
         }
+        n01 = fadd2(n01, e01);
+        n23 = fadd2(n23, e23);
+        d01 = fadd2(d01, h01);
+        d23 = fadd2(d23, h23);
         {
             float v[2][4] = {{f2lo(n01), f2hi(n01), f2lo(n23), f2hi(n23)},
                              {f2lo(d01), f2hi(d01), f2lo(d23), f2hi(d23)}};
@@ -313,18 +337,22 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
             }
             float c = S.colC[t.tid];
             if (den > 0.f) c = fminf(fmaxf(__fdiv_rn(num, den), kF16Min), kF16Max);
-            S.colC[t.tid] = c;
-            S.colG[t.tid] = __frcp_rn(c);
+            if (it + 1 < fit_iters) {
+                S.colC[t.tid] = c;
+                S.colG[t.tid] = __frcp_rn(c);
+            } else {
+                // storage precision of c; codes can clip only where max |X'| / c >= qmax + 1/2
+                const float cf = __half2float(__float2half_rn(c));
+                const float g = __frcp_rn(cf);
+                page_c[t.tid] = f16_bits(cf);
+                S.colG[t.tid] = g;
+                if (__fmul_rn(S.colX[t.tid], g) >= fqm + 0.5f) S.flags[2] = 1;
+            }
         }
         __syncthreads();
     }
-    // Storage precision of c, then the final codes with the stored scales.
-    if (t.tid < 128) {
-        const float cf = __half2float(__float2half_rn(S.colC[t.tid]));
-        page_c[t.tid] = f16_bits(cf);
-        S.colG[t.tid] = __frcp_rn(cf);
-    }
-    __syncthreads();
+    // Final codes with the stored scales.
+    const bool clip = S.flags[2] != 0;
     const uint64_t MB = f2s(kMagic + (float)(1 << (B - 1)));
 #pragma unroll
     for (int c = 0; c < 4; c += 2) {
@@ -332,11 +360,12 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         uint32_t ua[16], ub[16];
 #pragma unroll
         for (int r = 0; r < 16; r++) {
-            const uint64_t tq = fmul2(x2[r][c >> 1], g);
-            const uint64_t cl = f2(fminf(fmaxf(f2lo(tq), -fqm), fqm), fminf(fmaxf(f2hi(tq), -fqm), fqm));
-            const uint64_t uu = fadd2(cl, MB);             // bits: 0x4B400000 + (q + 2^(B-1))
-            ua[r] = __float_as_uint(f2lo(uu));
-            ub[r] = __float_as_uint(f2hi(uu));
+            uint64_t tq = fmul2(x2[r][c >> 1], g);
+            if (clip)
+                tq = f2(fminf(fmaxf(f2lo(tq), -fqm), fqm), fminf(fmaxf(f2hi(tq), -fqm), fqm));
+            const uint64_t uu = fadd2(tq, MB);              // bits: 0x4B400000 + (q + 2^(B-1))
+            ua[r] = (uint32_t)uu;
+            ub[r] = (uint32_t)(uu >> 32);
         }
         uint32_t wd[8];
         pack16<B>(ua, wd);
@@ -346,23 +375,25 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
     }
 }
 
-// FP16 pivot head: store fp16(X) (saturating) in band-major order.
-__device__ __forceinline__ void pack_pivot(const T &t, uint8_t *page, const uint64_t (&x2)[16][2]) {
+// FP16 pivot head: store fp16(a_i Z) (saturating) in band-major order.
+__device__ __forceinline__ void pack_pivot(const T &t, uint8_t *page, const uint64_t (&x2)[16][2],
+                                           float a) {
 #pragma unroll
     for (int c = 0; c < 4; c++) {
         uint32_t wd[8];
 #pragma unroll
         for (int r = 0; r < 16; r += 2) {
-            const float a = (c & 1) ? f2hi(x2[r][c >> 1]) : f2lo(x2[r][c >> 1]);
-            const float b = (c & 1) ? f2hi(x2[r + 1][c >> 1]) : f2lo(x2[r + 1][c >> 1]);
-            wd[r >> 1] = (uint32_t)f16_bits(f16_round_sat(a)) | ((uint32_t)f16_bits(f16_round_sat(b)) << 16);
+            const float za = (c & 1) ? f2hi(x2[r][c >> 1]) : f2lo(x2[r][c >> 1]);
+            const float zb = (c & 1) ? f2hi(x2[r + 1][c >> 1]) : f2lo(x2[r + 1][c >> 1]);
+            wd[r >> 1] = (uint32_t)f16_bits(f16_round_sat(a * za)) |
+                         ((uint32_t)f16_bits(f16_round_sat(a * zb)) << 16);
         }
         store_chunk<kPivot>(page + chunk_off<kPivot>(t.w, t.col(c)), wd);
     }
 }
 
-// Reconstruct S_hat into x2 (scaled per column: x = c_j q for integer heads,
-// the FP16 value for pivot heads); the row factor is applied by the caller.
+// Reconstruct the column-scaled codes c_j q_ij (exact in fp32) or the FP16
+// values of a pivot head; the row factor stays separate.
 template <int B>
 __device__ __forceinline__ void load_tile(const T &t, const uint8_t *page, uint64_t (&x2)[16][2]) {
     const uint16_t *page_c = (const uint16_t *)(page + 256);
@@ -380,13 +411,15 @@ __device__ __forceinline__ void load_tile(const T &t, const uint8_t *page, uint6
             }
         } else {
             const float ca = f16_val(page_c[t.col(c)]), cb = f16_val(page_c[t.col(c + 1)]);
-            constexpr float off = (float)(1 << (B - 1));
-            const uint64_t cc = f2(ca, cb), oc = f2(-off * ca, -off * cb);   // exact constants
+            // 0x4B400000 + u - 2^(B-1) is the float 1.5*2^23 + q; fma(f, c, -1.5*2^23 c)
+            // = c q exactly (c fp16, |q| <= 127: 19 significant bits; 1.5*2^23 c exact).
+            constexpr uint32_t kBias = 0x4B400000u - (1u << (B - 1));
+            const uint64_t cc = f2(ca, cb), oc = f2(-kMagic * ca, -kMagic * cb);
 #pragma unroll
             for (int r = 0; r < 16; r++) {
-                // c_j (u - off) with one rounding: fma(u, c_j, -off c_j), -off c_j exact
-                const uint64_t uf = f2((float)code_at<B>(wa, r), (float)code_at<B>(wb, r));
-                x2[r][c >> 1] = ffma2(uf, cc, oc);
+                const uint64_t fq = ((uint64_t)(code_at<B>(wb, r) + kBias) << 32) |
+                                    (uint64_t)(code_at<B>(wa, r) + kBias);
+                x2[r][c >> 1] = ffma2(fq, cc, oc);
             }
         }
     }
@@ -436,30 +469,44 @@ __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int it
 // One decode step of one head page staged in shared memory (width B).
 // `refill` runs once the stage's inputs are fully consumed (after the retrieval
 // reduction); the page itself is rewritten in place afterwards.
+//
+// With a_i = alpha r_i (> 0) and Z_ij = c_j q_ij + (beta k_i / a_i) delta_j the
+// update is X_ij = a_i Z_ij: one fma per element instead of two.
 template <int B, class Refill>
 __device__ __forceinline__ void decode_item(const T &t, const Smem &S, const Stage &st, float alpha,
                                             float beta, float *y_out, int fit_iters,
                                             const Refill &refill) {
     const uint16_t *page_r = (const uint16_t *)st.page;
-    // Row constants: a_i = alpha r_i (reconstruction and gate), kappa_i = k_i a_i,
-    // beta k_i, q_i.
-    if (t.tid < 128) {
-        const int i = t.tid;
-        const float a = B == kPivot ? alpha : alpha * f16_val(page_r[i]);
+    // Row constants of the warp's band (warp-local): a_i, kappa_i = k_i a_i,
+    // beta k_i / a_i, q_i a_i, as duplicated fp32 pairs.
+    if (t.l < 16) {
+        const int i = t.row(t.l);
+        const float a = fmaxf(B == kPivot ? alpha : alpha * f16_val(page_r[i]), 1e-30f);
         const float ki = st.k[i];
-        S.rowc[i] = make_float4(a, ki * a, beta * ki, st.q[i]);
+        const float kap = ki * a, bkp = __fdiv_rn(beta * ki, a), qa = st.q[i] * a;
+        S.rowc[2 * i] = make_float4(kap, kap, bkp, bkp);
+        S.rowc[2 * i + 1] = make_float4(qa, qa, a, a);
+        S.rowa[i] = a;
     }
     uint64_t x2[16][2];
     load_tile<B>(t, st.page, x2);
-    __syncthreads();
-    // Step 2a: retrieval u_j = sum_i k_i (D S_hat)_ij.
-    uint64_t u01 = 0, u23 = 0;
+    __syncwarp();
+    // Step 2a: retrieval u_j = sum_i k_i a_i (c_j q_ij).
+    uint64_t u01 = 0, u23 = 0, v01 = 0, v23 = 0;
 #pragma unroll
     for (int r = 0; r < 16; r++) {
-        const uint64_t kap = f2s(S.rowc[t.row(r)].y);
-        u01 = ffma2(kap, x2[r][0], u01);
-        u23 = ffma2(kap, x2[r][1], u23);
+        const uint4 rc = *(const uint4 *)&S.rowc[2 * t.row(r)];
+        const uint64_t kap = ((uint64_t)rc.y << 32) | rc.x;
+        if (r & 1) {
+            v01 = ffma2(kap, x2[r][0], v01);
+            v23 = ffma2(kap, x2[r][1], v23);
+        } else {
+            u01 = ffma2(kap, x2[r][0], u01);
+            u23 = ffma2(kap, x2[r][1], u23);
+        }
     }
+    u01 = fadd2(u01, v01);
+    u23 = fadd2(u23, v23);
     {
         float v[1][4] = {{f2lo(u01), f2hi(u01), f2lo(u23), f2hi(u23)}};
         cols_to_red<1>(t, S.red, v);
@@ -473,22 +520,31 @@ __device__ __forceinline__ void decode_item(const T &t, const Smem &S, const Sta
     }
     refill();
     __syncthreads();
-    // Step 2b-3: X = a_i (c_j q_ij) + beta k_i delta_j; readout partials q_i X_ij.
+    // Step 2b-3: Z = c q + (beta k / a) delta; readout partials q_i a_i Z_ij.
     const uint64_t dl01 = f2(S.colD[t.col(0)], S.colD[t.col(1)]);
     const uint64_t dl23 = f2(S.colD[t.col(2)], S.colD[t.col(3)]);
-    uint64_t y01 = 0, y23 = 0;
+    uint64_t y01 = 0, y23 = 0, z01 = 0, z23 = 0;
     float rs[16];
 #pragma unroll
     for (int r = 0; r < 16; r++) {
-        const float4 rc = S.rowc[t.row(r)];
-        const uint64_t a = f2s(rc.x), bk = f2s(rc.z), qi = f2s(rc.w);
-        x2[r][0] = ffma2(a, x2[r][0], fmul2(bk, dl01));
-        x2[r][1] = ffma2(a, x2[r][1], fmul2(bk, dl23));
-        y01 = ffma2(qi, x2[r][0], y01);
-        y23 = ffma2(qi, x2[r][1], y23);
-        rs[r] = fabsf(f2lo(x2[r][0])) + fabsf(f2hi(x2[r][0])) + fabsf(f2lo(x2[r][1])) +
-                fabsf(f2hi(x2[r][1]));
+        const uint4 rc = *(const uint4 *)&S.rowc[2 * t.row(r)];
+        const uint4 rq = *(const uint4 *)&S.rowc[2 * t.row(r) + 1];
+        const uint64_t bkp = ((uint64_t)rc.w << 32) | rc.z;
+        const uint64_t qa = ((uint64_t)rq.y << 32) | rq.x;
+        x2[r][0] = ffma2(bkp, dl01, x2[r][0]);
+        x2[r][1] = ffma2(bkp, dl23, x2[r][1]);
+        if (r & 1) {
+            z01 = ffma2(qa, x2[r][0], z01);
+            z23 = ffma2(qa, x2[r][1], z23);
+        } else {
+            y01 = ffma2(qa, x2[r][0], y01);
+            y23 = ffma2(qa, x2[r][1], y23);
+        }
+        rs[r] = (fabsf(f2lo(x2[r][0])) + fabsf(f2hi(x2[r][0]))) +
+                (fabsf(f2lo(x2[r][1])) + fabsf(f2hi(x2[r][1])));
     }
+    y01 = fadd2(y01, z01);
+    y23 = fadd2(y23, z23);
     const float yp[4] = {f2lo(y01), f2hi(y01), f2lo(y23), f2hi(y23)};
     if (B == kPivot) {
         float v[1][4] = {{yp[0], yp[1], yp[2], yp[3]}};
@@ -500,11 +556,11 @@ __device__ __forceinline__ void decode_item(const T &t, const Smem &S, const Sta
             for (int wv = 0; wv < 8; wv++) s += S.red[wv * 128 + t.tid];
             y_out[t.tid] = s;
         }
-        pack_pivot(t, st.page, x2);
+        pack_pivot(t, st.page, x2, fmaxf(alpha, 1e-30f));
         return;
     }
     // Steps 4-6: refit and repack in place.
-    fit_pack<B>(t, S, st.page, st.w2, st.wis, x2, rs, yp, true, y_out, fit_iters);
+    fit_pack<B>(t, S, st.page, st.w2, st.wis, S.rowa, x2, rs, yp, true, y_out, fit_iters);
 }
 
 __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a) {
@@ -634,11 +690,11 @@ __device__ __forceinline__ void quantize_item(const T &t, const Smem &S, uint8_t
         rs[r] = fabsf(a) + fabsf(b) + fabsf(c) + fabsf(d);
     }
     if (B == kPivot) {
-        pack_pivot(t, page, x2);
+        pack_pivot(t, page, x2, 1.f);
         return;
     }
     const float none[4] = {0.f, 0.f, 0.f, 0.f};
-    fit_pack<B>(t, S, page, w2, wis, x2, rs, none, false, nullptr, fit_iters);
+    fit_pack<B>(t, S, page, w2, wis, nullptr, x2, rs, none, false, nullptr, fit_iters);
 }
 
 __global__ void __launch_bounds__(kThreads, 2) quantize_heads_kernel(PoolArgs a) {
