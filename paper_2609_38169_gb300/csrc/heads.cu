@@ -29,7 +29,7 @@ constexpr int kVecBytes = 5 * 512;                     // q k v w2 wis per stage
 constexpr int kOffBars = 0;                            // uint64 [8]
 constexpr int kOffFlags = 64;                          // int [16]
 constexpr int kOffRed = 128;                           // float [2][8][128]
-constexpr int kOffCol = kOffRed + 2 * 8 * 128 * 4;     // float [4][128]
+constexpr int kOffCol = kOffRed + 2 * 8 * 128 * 4;     // float [4][128] (colX and paired G, D)
 constexpr int kOffRowC = kOffCol + 4 * 128 * 4;        // float4 [2][128]: kappa,kappa,bk',bk' | qa,qa,a,a
 constexpr int kOffRowF = kOffRowC + 256 * 16;          // float4 [128]: rho a, rho a, alpha_ls, alpha_ls
 constexpr int kOffRowA = kOffRowF + 128 * 16;          // float [128]: a_i
@@ -78,6 +78,8 @@ struct Stage {
         wis = q + 512;
     }
 };
+
+constexpr int kProducer = kThreads - 32;              // lane 0 of the last warp issues copies
 
 struct T {   // thread coordinates
     int tid, w, l;
@@ -197,6 +199,16 @@ __device__ __forceinline__ float warp_row_sums(float (&v)[16], int l, int &row_o
     return a1;
 }
 
+// Column vectors are kept in "pair" order so a thread loads the values of its
+// column pairs (l, l+32) and (l+64, l+96) as one 64-bit word each.
+__device__ __forceinline__ int pair_idx(int j) {      // column j -> float index in the pair array
+    const int m = j >> 6, rem = j & 63;                 // rem = l or l + 32
+    return (m * 32 + (rem & 31)) * 2 + (rem >> 5);
+}
+__device__ __forceinline__ uint64_t load_pair(const float *v, int l, int m) {
+    return *(const uint64_t *)&v[(m * 32 + l) * 2];
+}
+
 // Cross-warp column reduction of NR values per thread column (4 columns per
 // thread, 8 warps); results land in out[k][128] for threads 0..127 to use.
 template <int NR>
@@ -277,14 +289,14 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         if (c0 > kF16Max) S.flags[1] = 1;                 // start capped: codes may clip
         const float c = fminf(fmaxf(c0, kF16Min), kF16Max);
         S.colC[t.tid] = c;
-        S.colG[t.tid] = __frcp_rn(c);
+        S.colG[pair_idx(t.tid)] = __frcp_rn(c);
         S.colX[t.tid] = mx;                               // max_i |X'_ij|
-        if (with_y) {
-            float s = S.red[8 * 128 + t.tid];
+    } else if (with_y) {
+        const int j = t.tid - 128;
+        float s = S.red[8 * 128 + j];
 #pragma unroll
-            for (int wv = 1; wv < 8; wv++) s += S.red[(8 + wv) * 128 + t.tid];
-            y_out[t.tid] = s;
-        }
+        for (int wv = 1; wv < 8; wv++) s += S.red[(8 + wv) * 128 + j];
+        y_out[j] = s;
     }
     __syncthreads();
     // Fixed-code least-squares updates: c_j = sum alpha_i q_ij X'_ij / sum alpha_i q_ij^2
@@ -292,8 +304,8 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
     const uint64_t M2 = f2s(kMagic), nM2 = f2s(-kMagic);
     for (int it = 0; it < fit_iters; it++) {
         const bool clip = it > 0 || S.flags[1];
-        const uint64_t g01 = f2(S.colG[t.col(0)], S.colG[t.col(1)]);
-        const uint64_t g23 = f2(S.colG[t.col(2)], S.colG[t.col(3)]);
+        const uint64_t g01 = load_pair(S.colG, t.l, 0);
+        const uint64_t g23 = load_pair(S.colG, t.l, 1);
         uint64_t n01 = 0, n23 = 0, d01 = 0, d23 = 0, e01 = 0, e23 = 0, h01 = 0, h23 = 0;
 #pragma unroll
         for (int r = 0; r < 16; r++) {
@@ -335,17 +347,18 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
                 num += S.red[wv * 128 + t.tid];
                 den += S.red[(8 + wv) * 128 + t.tid];
             }
+            // num and den carry fp32 summation error already; a 2-ulp quotient adds nothing
             float c = S.colC[t.tid];
-            if (den > 0.f) c = fminf(fmaxf(__fdiv_rn(num, den), kF16Min), kF16Max);
+            if (den > 0.f) c = fminf(fmaxf(__fdividef(num, den), kF16Min), kF16Max);
             if (it + 1 < fit_iters) {
                 S.colC[t.tid] = c;
-                S.colG[t.tid] = __frcp_rn(c);
+                S.colG[pair_idx(t.tid)] = __frcp_rn(c);
             } else {
                 // storage precision of c; codes can clip only where max |X'| / c >= qmax + 1/2
                 const float cf = __half2float(__float2half_rn(c));
                 const float g = __frcp_rn(cf);
                 page_c[t.tid] = f16_bits(cf);
-                S.colG[t.tid] = g;
+                S.colG[pair_idx(t.tid)] = g;
                 if (__fmul_rn(S.colX[t.tid], g) >= fqm + 0.5f) S.flags[2] = 1;
             }
         }
@@ -356,7 +369,7 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
     const uint64_t MB = f2s(kMagic + (float)(1 << (B - 1)));
 #pragma unroll
     for (int c = 0; c < 4; c += 2) {
-        const uint64_t g = f2(S.colG[t.col(c)], S.colG[t.col(c + 1)]);
+        const uint64_t g = load_pair(S.colG, t.l, c >> 1);
         uint32_t ua[16], ub[16];
 #pragma unroll
         for (int r = 0; r < 16; r++) {
@@ -516,13 +529,13 @@ __device__ __forceinline__ void decode_item(const T &t, const Smem &S, const Sta
         float s = 0.f;
 #pragma unroll
         for (int wv = 0; wv < 8; wv++) s += S.red[wv * 128 + t.tid];
-        S.colD[t.tid] = st.v[t.tid] - s;                    // delta_j = v_j - u_j
+        S.colD[pair_idx(t.tid)] = st.v[t.tid] - s;          // delta_j = v_j - u_j
     }
     refill();
     __syncthreads();
     // Step 2b-3: Z = c q + (beta k / a) delta; readout partials q_i a_i Z_ij.
-    const uint64_t dl01 = f2(S.colD[t.col(0)], S.colD[t.col(1)]);
-    const uint64_t dl23 = f2(S.colD[t.col(2)], S.colD[t.col(3)]);
+    const uint64_t dl01 = load_pair(S.colD, t.l, 0);
+    const uint64_t dl23 = load_pair(S.colD, t.l, 1);
     uint64_t y01 = 0, y23 = 0, z01 = 0, z23 = 0;
     float rs[16];
 #pragma unroll
@@ -575,17 +588,20 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
         S.hbytes[h] = a.tab.head_bytes[h];
         S.hbits[h] = a.tab.head_bits[h];
     }
-    if (t.tid == 0) {
+    if (t.tid == kProducer) {
         for (int s = 0; s < S_n; s++) mbar_init(&S.bars[s], 1);
         mbar_init_fence();
     }
     __syncthreads();
-    if (t.tid == 0) {
+    if (t.tid == kProducer) {
         for (int s = 0; s < S_n; s++) {
             const int item = first + s * G;
             if (item < a.items) issue(a, S, item, a.slots[item / a.Hv], s);
         }
     }
+    // With three or more stages a stage is refilled two items after its own item
+    // (its store has long finished reading it); with two stages, one item after.
+    const int lag = S_n >= 3 ? 2 : 1;
     // scalars of the current item; the next item's are fetched one iteration ahead
     int b = first / a.Hv, h = first - b * a.Hv;
     int slot = a.slots[b];
@@ -606,16 +622,17 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
             nalpha = a.gate[(size_t)nb * a.Hv + nh];
             nbeta = a.beta[(size_t)nb * a.Hv + nh];
         }
-        const int iitem = first + (n - 1 + S_n) * G;
+        const int iitem = first + (n - lag + S_n) * G;
         int islot = -1;
-        if (t.tid == 0 && iitem < a.items) islot = a.slots[iitem / a.Hv];
+        if (t.tid == kProducer && n >= lag && iitem < a.items) islot = a.slots[iitem / a.Hv];
 
         const bool ok = mbar_wait(&S.bars[s], parity, kWaitCycles);
         if (__syncthreads_or(!ok)) {
-            if (t.tid == 0) {
+            if (t.tid == kProducer) {
                 raise_error(a.err, STEPQ_ERR_TIMEOUT);
-                // drain this CTA's copies still in flight, again with a bound
-                for (int m = n; m < n + S_n - 1 + (n == 0 ? 1 : 0); m++) {
+                // drain this CTA's copies still in flight (items n .. issued), with a bound
+                const int last = n < lag ? S_n - 1 : n - 1 - lag + S_n;
+                for (int m = n; m <= last; m++) {
                     if (first + m * G >= a.items) break;
                     mbar_wait(&S.bars[m % S_n], (uint32_t)(m / S_n) & 1u, kWaitCycles);
                 }
@@ -629,9 +646,10 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
         // Refill the stage of the previous item (its store was committed one item
         // ago) with the item S-1 ahead of it: S-1 items stay in flight.
         const auto refill = [&]() {
-            if (t.tid == 0 && n > 0 && iitem < a.items) {
-                bulk_wait_read_all();
-                issue(a, S, iitem, islot, (n - 1) % S_n);
+            if (t.tid == kProducer && n >= lag && iitem < a.items) {
+                if (lag == 2) bulk_wait_read_all_but_one();
+                else bulk_wait_read_all();
+                issue(a, S, iitem, islot, (n - lag) % S_n);
             }
         };
         if (valid) {
@@ -647,7 +665,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
             refill();
         }
         __syncthreads();                                 // the page in stage s is final
-        if (t.tid == 0) {
+        if (t.tid == kProducer) {
             if (valid) {
                 fence_async_smem();
                 bulk_store(a.pool + (uint64_t)slot * a.stride + S.hoff[h], st.page, S.hbytes[h]);
@@ -656,7 +674,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
         }
         b = nb; h = nh; slot = nslot; alpha = nalpha; beta = nbeta;
     }
-    if (t.tid == 0) bulk_wait_all();
+    if (t.tid == kProducer) bulk_wait_all();
 }
 
 // ---------------------------------------------------------- pack / unpack
