@@ -219,6 +219,21 @@ stepq_status stepq_calib_distortion(const stepq_config *cfg, int layer, const fl
 stepq_status stepq_validate_slots(const int32_t *slots, int B, int pool_slots, uint32_t *scratch,
                                   int32_t *status_out, stepq_stream_t stream);
 
+/* The same check for callers that cannot allocate device memory and have no
+ * spare scratch buffer to pass -- for example code running where a host
+ * framework owns every device allocation, or on a path where cudaMalloc's
+ * implicit synchronisation is not acceptable. The paper has no counterpart;
+ * this entry point allocates nothing.
+ * The bitmap lives in a file-scope device array sized for pool_slots up to
+ * 1,048,576 (128 KiB, kept by every GPU that loads the library until the
+ * process exits); larger pools return STEPQ_ERR_UNSUPPORTED before any work.
+ * The first call on a device looks up the array's device address (set-up that
+ * should happen before any stream capture). Every call shares the array and
+ * clears the part it uses first; calls that overlap on the GPU race with each
+ * other. status_out: device int32, as for stepq_validate_slots. */
+stepq_status stepq_validate_slots_noalloc(const int32_t *slots, int B, int pool_slots,
+                                          int32_t *status_out, stepq_stream_t stream);
+
 /* Read and clear the sticky device error of the current device (synchronises
  * `stream`): STEPQ_OK, or the first error a kernel raised. */
 stepq_status stepq_device_error(stepq_stream_t stream);

@@ -301,6 +301,17 @@ def stepq_validate_slots(slots, pool_slots: int, scratch, status_out, stream=Non
           "stepq_validate_slots")
 
 
+def stepq_validate_slots_noalloc(slots, pool_slots: int, status_out, stream=None):
+    """stepq_validate_slots without a scratch argument: the library keeps the
+    bitmap in a fixed device array (pool_slots <= 1,048,576) and allocates nothing."""
+    import torch
+    check(_lib.lib().stepq_validate_slots_noalloc(_dev_ptr(slots, torch.int32), slots.numel(),
+                                                  int(pool_slots),
+                                                  _dev_ptr(status_out, torch.int32),
+                                                  _stream(stream)),
+          "stepq_validate_slots_noalloc")
+
+
 def stepq_device_error(stream=None) -> int:
     return int(_lib.lib().stepq_device_error(_stream(stream)))
 

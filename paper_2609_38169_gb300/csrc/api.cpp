@@ -198,6 +198,12 @@ extern "C" stepq_status stepq_validate_slots(const int32_t *slots, int B, int po
     return launch_validate_slots(slots, B, pool_slots, scratch, status_out, (cudaStream_t)stream);
 }
 
+extern "C" stepq_status stepq_validate_slots_noalloc(const int32_t *slots, int B, int pool_slots,
+                                                     int32_t *status_out, stepq_stream_t stream) {
+    if ((B > 0 && !slots) || B < 0 || pool_slots <= 0 || !status_out) return STEPQ_ERR_ARG;
+    return launch_validate_slots_static(slots, B, pool_slots, status_out, (cudaStream_t)stream);
+}
+
 extern "C" stepq_status stepq_device_error(stepq_stream_t stream) {
     return read_device_error((cudaStream_t)stream);
 }

@@ -56,4 +56,42 @@ stepq_status launch_validate_slots(const int32_t *slots, int B, int pool_slots,
     return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;
 }
 
+// ---- slot validation without allocation ----
+// For callers that cannot allocate device memory and have no spare scratch to
+// pass: the bitmap lives in this file-scope array, which every GPU that loads
+// the library keeps for the life of the process.
+constexpr int kStaticSlotMax = 1 << 20;                       // pool slots covered (128 KiB)
+static __device__ __align__(256) uint32_t g_slot_bitmap[kStaticSlotMax / 32];
+
+// Device address of the array on the current device, looked up once per device.
+// Host code must not hand the symbol itself to a kernel: on the host it only
+// names a stand-in, not device memory.
+static uint32_t *static_bitmap(stepq_status *st) {
+    static uint32_t *addr[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+        *st = STEPQ_ERR_CUDA;
+        return nullptr;
+    }
+    if (!addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_slot_bitmap) != cudaSuccess || !p) {
+            *st = STEPQ_ERR_CUDA;
+            return nullptr;
+        }
+        addr[dev] = (uint32_t *)p;
+    }
+    return addr[dev];
+}
+
+stepq_status launch_validate_slots_static(const int32_t *slots, int B, int pool_slots,
+                                          int32_t *status, cudaStream_t s) {
+    if (pool_slots > kStaticSlotMax) return STEPQ_ERR_UNSUPPORTED;
+    stepq_status st = STEPQ_OK;
+    uint32_t *bitmap = static_bitmap(&st);
+    if (!bitmap) return st;
+    // the same validator; it clears the (pool_slots + 31) / 32 words it uses first
+    return launch_validate_slots(slots, B, pool_slots, bitmap, status, s);
+}
+
 }  // namespace stepq

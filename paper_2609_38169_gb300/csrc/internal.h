@@ -123,6 +123,8 @@ stepq_status launch_calib_distortion(const stepq_config *cfg, int layer, const f
                                      double *acc, cudaStream_t s);
 stepq_status launch_validate_slots(const int32_t *slots, int B, int pool_slots,
                                    uint32_t *scratch, int32_t *status, cudaStream_t s);
+stepq_status launch_validate_slots_static(const int32_t *slots, int B, int pool_slots,
+                                          int32_t *status, cudaStream_t s);
 stepq_status read_device_error(cudaStream_t s);
 unsigned int *device_error_word();   // address of the current device's sticky error word
 
