@@ -94,6 +94,19 @@ def _recorded_traffic(units_per_launch: int):
         return None
 
 
+def reduce_over_ranks(total_ms: float, units: float, world: int, device=None):
+    """Max of the timed region over ranks and the whole-job rate: every rank runs
+    its own replica, so all ranks' units count over the slowest rank's time."""
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([float(total_ms)], dtype=torch.float64,
+                         device=device if device is not None else "cpu")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    return total_ms, world * units / (total_ms / 1e3)
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -160,7 +173,7 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=40)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="stepq", choices=["stepq", "reference"])
     ap.add_argument("--no-baselines", action="store_true")
@@ -281,14 +294,9 @@ def main():
     clocks.start()
     total_ms, launch_ms = timed(step_stepq, args.steps, args.warmup, per_launch=True, name="stepq_decode")
     clk = clocks.stop()
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
     assert P.stepq_device_error() == 0
     units_per_step = L * B * Hv
-    value = world * units_per_step * args.steps / (total_ms / 1e3)
+    total_ms, value = reduce_over_ranks(total_ms, units_per_step * args.steps, world, dev)
 
     # algorithmic bytes per launch: each head page read and written once, plus
     # q, k (per key head), v, beta, gate read and y written
@@ -325,15 +333,10 @@ def main():
                                 pool_slots=wl.pool_slots)
         h_y.copy_(y, non_blocking=True)
 
-    e2e_ms, _ = timed(step_e2e, max(3, args.steps // 2), 2, name="stepq_e2e")
     e2e_steps = max(3, args.steps // 2)
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e = {"value": world * units_per_step * e2e_steps / (e2e_ms / 1e3), "unit": UNIT,
-           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+    e2e_ms, _ = timed(step_e2e, e2e_steps, 2, name="stepq_e2e")
+    e2e_ms, e2e_value = reduce_over_ranks(e2e_ms, units_per_step * e2e_steps, world, dev)
+    e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     baselines = {}
     if not args.no_baselines:
