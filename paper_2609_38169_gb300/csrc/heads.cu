@@ -2,15 +2,19 @@
 // the pack/unpack kernels for head pages stored in band-major order.
 //
 // Tile mapping: warp w owns the band of key rows 16w..16w+15; lane l owns the
-// value columns l, l+32, l+64, l+96. A thread holds a 16 x 4 register tile, so
-// every column reduction needs only one cross-warp step and the single row
-// reduction (m_i) stays inside a warp. In the band-major page a thread's 16
-// codes of one column are one 2b-byte chunk, and consecutive lanes read
-// consecutive chunks (no shared-memory bank conflicts).
+// value columns l, l+32, l+64, l+96. A thread holds a 16 x 4 register tile as
+// eight row pairs (rows 2m, 2m+1 of its band) per column, each pair one packed
+// f32x2 register: per-row constants of a row pair are adjacent in shared
+// memory (one 128-bit broadcast load serves two pairs), and the two codes of a
+// pair are adjacent in the band-major chunk. Every column reduction needs one
+// cross-warp step and the single row reduction (m_i) stays inside a warp. In
+// the page a thread's 16 codes of one column are one 2b-byte chunk and
+// consecutive lanes read consecutive chunks (no shared-memory bank conflicts).
 //
 // Decode pipeline (App. C.3 steps 1-7 per head): each persistent CTA walks its
-// (slot, head) items; one thread keeps up to S-1 pages in flight with bulk
-// copies completing on per-stage mbarriers, the CTA updates and refits the
+// (head, slot) items, head-major so that concurrently resident CTAs mostly run
+// the code of one head width; one thread keeps up to S-1 pages in flight with
+// bulk copies completing on per-stage mbarriers, the CTA updates and refits the
 // page in place in shared memory, and a bulk store writes it back. Every wait
 // is bounded: a stalled copy raises STEPQ_ERR_TIMEOUT and the CTA drains its
 // own copies before returning.
@@ -23,45 +27,55 @@ namespace hk {
 
 constexpr long long kWaitCycles = 2000000000LL;      // ~1 s at 2 GHz
 constexpr float kMagic = 12582912.0f;                  // 1.5 * 2^23: rint by addition
+constexpr uint32_t kMagicBits = 0x4B400000u;           // its bit pattern (low 22 bits zero)
 constexpr int kVecBytes = 5 * 512;                     // q k v w2 wis per stage
 
 // ------------------------------------------------------------ shared layout
 constexpr int kOffBars = 0;                            // uint64 [8]
 constexpr int kOffFlags = 64;                          // int [16]
-constexpr int kOffRed = 128;                           // float [2][8][128]
-constexpr int kOffCol = kOffRed + 2 * 8 * 128 * 4;     // float [4][128] (colX and paired G, D)
-constexpr int kOffRowC = kOffCol + 4 * 128 * 4;        // float4 [2][128]: kappa,kappa,bk',bk' | qa,qa,a,a
-constexpr int kOffRowF = kOffRowC + 256 * 16;          // float4 [128]: rho a, rho a, alpha_ls, alpha_ls
-constexpr int kOffRowA = kOffRowF + 128 * 16;          // float [128]: a_i
+constexpr int kOffRed = 128;                           // float [3][8][128] cross-warp partials
+constexpr int kOffColC = kOffRed + 3 * 8 * 128 * 4;    // float [128] c_j (start / iterate)
+constexpr int kOffColX = kOffColC + 512;               // float [128] max_i |X'_ij|
+constexpr int kOffColM = kOffColX + 512;               // u32 [128] bits of max_i |X'_ij| (atomic)
+constexpr int kOffColD = kOffColM + 512;               // float2 [128] (delta_j, delta_j)
+constexpr int kOffColG = kOffColD + 1024;              // float2 [128] (1/c_j, 1/c_j)
+constexpr int kOffRows = kOffColG + 1024;              // float [6][128] per-row constants
 constexpr int kMaxHv = 256;                            // value heads per layer (launch check)
-constexpr int kOffHead = kOffRowA + 128 * 4;           // u64 off[256] | u32 bytes[256] | u8 bits[256]
-constexpr int kOffStages = (kOffHead + kMaxHv * 13 + 127) / 128 * 128;
+constexpr int kOffHead = kOffRows + 6 * 512;           // u64 off | u32 bytes | u8 bits | u8 key head
+constexpr int kOffStages = (kOffHead + kMaxHv * 14 + 127) / 128 * 128;
 
 struct Smem {
     uint64_t *bars;
     int *flags;
-    float *red, *colC, *colG, *colD, *colX;
-    float4 *rowc;
-    float4 *rowf;
-    float *rowa;
+    float *red, *colC, *colX;
+    uint32_t *colM;
+    float2 *colD, *colG;
+    // per-row constants: kappa_i = k_i a_i, beta k_i / a_i, q_i a_i, a_i,
+    // rho_i a_i and the least-squares weight alpha_i = w_i^2 r_i^2
+    float *rKap, *rBkp, *rQa, *rA, *rRho, *rAl;
     uint64_t *hoff;
     uint32_t *hbytes;
-    uint8_t *hbits;
+    uint8_t *hbits, *hkey;
     uint8_t *stages;
     __device__ __forceinline__ explicit Smem(uint8_t *s) {
         bars = (uint64_t *)(s + kOffBars);
         flags = (int *)(s + kOffFlags);
         red = (float *)(s + kOffRed);
-        colC = (float *)(s + kOffCol);
-        colG = colC + 128;
-        colD = colC + 256;
-        colX = colC + 384;
-        rowc = (float4 *)(s + kOffRowC);
-        rowf = (float4 *)(s + kOffRowF);
-        rowa = (float *)(s + kOffRowA);
+        colC = (float *)(s + kOffColC);
+        colX = (float *)(s + kOffColX);
+        colM = (uint32_t *)(s + kOffColM);
+        colD = (float2 *)(s + kOffColD);
+        colG = (float2 *)(s + kOffColG);
+        rKap = (float *)(s + kOffRows);
+        rBkp = rKap + 128;
+        rQa = rKap + 256;
+        rA = rKap + 384;
+        rRho = rKap + 512;
+        rAl = rKap + 640;
         hoff = (uint64_t *)(s + kOffHead);
         hbytes = (uint32_t *)(s + kOffHead + kMaxHv * 8);
         hbits = s + kOffHead + kMaxHv * 12;
+        hkey = s + kOffHead + kMaxHv * 13;
         stages = s + kOffStages;
     }
 };
@@ -92,6 +106,16 @@ struct T {   // thread coordinates
     __device__ __forceinline__ int col(int c) const { return l + 32 * c; }
 };
 
+// Row-pair constants m = 2p, 2p+1 of the warp's band from one 128-bit load.
+__device__ __forceinline__ void row_pairs(const float *v, const T &t, int p, uint64_t &lo, uint64_t &hi) {
+    const uint4 q = *(const uint4 *)&v[t.row(4 * p)];
+    lo = u2pair(q.x, q.y);
+    hi = u2pair(q.z, q.w);
+}
+__device__ __forceinline__ uint64_t col_pair(const float2 *v, int j) {
+    return *(const uint64_t *)&v[j];
+}
+
 // Byte offset of the band-major chunk (band w, column j) in a head page.
 template <int B>
 __device__ __forceinline__ int chunk_off(int w, int j) {
@@ -120,14 +144,6 @@ __device__ __forceinline__ void load_chunk(const uint8_t *p, uint32_t (&wd)[8]) 
 }
 
 template <int B>
-__device__ __forceinline__ uint32_t code_at(const uint32_t (&wd)[8], int r) {
-    const int bit = r * B, wi = bit >> 5, sh = bit & 31;
-    constexpr uint32_t mask = (1u << B) - 1u;
-    if (sh + B <= 32) return (wd[wi] >> sh) & mask;
-    return __funnelshift_r(wd[wi], wd[wi + 1], sh) & mask;
-}
-
-template <int B>
 __device__ __forceinline__ void store_chunk(uint8_t *p, const uint32_t (&wd)[8]) {
     if (B == 2) {
         *(uint32_t *)p = wd[0];
@@ -144,28 +160,72 @@ __device__ __forceinline__ void store_chunk(uint8_t *p, const uint32_t (&wd)[8])
     }
 }
 
-// 16 offset-binary codes (low B bits of u[r]) into the chunk words.
+// Scale of the high code of a pair as placed by code_pair (2^B, or 1 for B = 8).
 template <int B>
-__device__ __forceinline__ void pack16(const uint32_t (&u)[16], uint32_t (&wd)[8]) {
+__host__ __device__ constexpr float hi_scale() { return B == 8 ? 1.0f : 1.0f / (float)(1 << B); }
+
+// Codes 2m and 2m+1 of a chunk as the bit patterns of the floats
+// 1.5*2^23 + u_lo and 1.5*2^23 + u_hi * 2^B (B = 8: both at the bottom): the
+// codes are dropped into the zero low mantissa bits of the constant, one logic
+// op each (after at most one shift per pair).
+template <int B>
+__device__ __forceinline__ uint64_t code_pair(const uint32_t (&wd)[8], int m) {
+    if (B == 8) {
+        const uint32_t w = wd[m >> 1];
+        const uint32_t sel = 0x7650u + 2u * (uint32_t)(m & 1);
+        return u2pair(__byte_perm(w, kMagicBits, sel), __byte_perm(w, kMagicBits, sel + 1u));
+    }
+    constexpr uint32_t mask = (1u << B) - 1u;
+    const int p = 2 * m * B, k = p >> 5, s = p & 31;
+    uint32_t win;
+    if (s == 0)
+        win = wd[k];
+    else if (s + 2 * B <= 32)
+        win = wd[k] >> s;
+    else
+        win = __funnelshift_r(wd[k], wd[k + 1], s);
+    return u2pair(and_or(win, mask, kMagicBits), and_or(win, mask << B, kMagicBits));
+}
+
+// Sum over the 16 codes of the chunk of (0x4B400000 << s) and of the parts
+// shifted into the next word, i.e. what pack_codes adds besides the codes.
+__host__ __device__ constexpr uint32_t pack_bias(int B, int k) {
+    uint32_t b = 0;
+    for (int r = 0; r < 16; r++) {
+        const int p = r * B, kk = p >> 5, s = p & 31;
+        if (kk == k) b += kMagicBits << s;
+        if (s + B > 32 && kk + 1 == k) b += kMagicBits >> (32 - s);
+    }
+    return b;
+}
+
+// 16 offset-binary codes given as the float bit patterns 0x4B400000 | u_r,
+// packed LSB-first into the chunk words. The high bits are the same constant
+// for every code, so each word is the plain sum of the shifted patterns minus
+// the shifted constants (mod 2^32): one shift-add per code.
+template <int B>
+__device__ __forceinline__ void pack_codes(const uint32_t (&f)[16], uint32_t (&wd)[8]) {
     if (B == 8) {
 #pragma unroll
         for (int t = 0; t < 4; t++) {
-            const uint32_t lo = __byte_perm(u[4 * t], u[4 * t + 1], 0x0040);
-            const uint32_t hi = __byte_perm(u[4 * t + 2], u[4 * t + 3], 0x0040);
+            const uint32_t lo = __byte_perm(f[4 * t], f[4 * t + 1], 0x0040);
+            const uint32_t hi = __byte_perm(f[4 * t + 2], f[4 * t + 3], 0x0040);
             wd[t] = __byte_perm(lo, hi, 0x5410);
         }
         return;
     }
-    constexpr uint32_t mask = (1u << B) - 1u;
+    constexpr int NW = B / 2;
+    uint32_t acc[NW];
 #pragma unroll
-    for (int t = 0; t < B / 2; t++) wd[t] = 0u;
+    for (int k = 0; k < NW; k++) acc[k] = 0u - pack_bias(B, k);
 #pragma unroll
     for (int r = 0; r < 16; r++) {
-        const uint32_t v = u[r] & mask;
-        const int bit = r * B, wi = bit >> 5, sh = bit & 31;
-        wd[wi] |= v << sh;
-        if (sh + B > 32) wd[wi + 1] |= v >> (32 - sh);
+        const int p = r * B, k = p >> 5, s = p & 31;
+        acc[k] += f[r] << s;
+        if (s + B > 32) acc[k + 1] += f[r] >> (32 - s);
     }
+#pragma unroll
+    for (int k = 0; k < NW; k++) wd[k] = acc[k];
 }
 
 // Sum of 16 per-row partials over the 32 lanes of a warp (reduce-scatter): lane
@@ -199,37 +259,94 @@ __device__ __forceinline__ float warp_row_sums(float (&v)[16], int l, int &row_o
     return a1;
 }
 
-// Column vectors are kept in "pair" order so a thread loads the values of its
-// column pairs (l, l+32) and (l+64, l+96) as one 64-bit word each.
-__device__ __forceinline__ int pair_idx(int j) {      // column j -> float index in the pair array
-    const int m = j >> 6, rem = j & 63;                 // rem = l or l + 32
-    return (m * 32 + (rem & 31)) * 2 + (rem >> 5);
-}
-__device__ __forceinline__ uint64_t load_pair(const float *v, int l, int m) {
-    return *(const uint64_t *)&v[(m * 32 + l) * 2];
-}
-
 // Cross-warp column reduction of NR values per thread column (4 columns per
-// thread, 8 warps); results land in out[k][128] for threads 0..127 to use.
+// thread, 8 warps) into partial region `reg0` and the following ones.
 template <int NR>
-__device__ __forceinline__ void cols_to_red(const T &t, float *red, const float (&v)[NR][4]) {
+__device__ __forceinline__ void cols_to_red(const T &t, float *red, int reg0, const float (&v)[NR][4]) {
 #pragma unroll
     for (int k = 0; k < NR; k++)
 #pragma unroll
-        for (int c = 0; c < 4; c++) red[(k * 8 + t.w) * 128 + t.col(c)] = v[k][c];
+        for (int c = 0; c < 4; c++) red[((reg0 + k) * 8 + t.w) * 128 + t.col(c)] = v[k][c];
+}
+__device__ __forceinline__ float pair_sum(uint64_t v) { return f2lo(v) + f2hi(v); }
+
+// Per-row sums over the thread's 4 columns of |value|, for the row pair's
+// low (even) and high (odd) rows.
+__device__ __forceinline__ void abs_row_sums(const uint64_t (&x)[4], float &lo, float &hi) {
+    lo = (fabsf(f2lo(x[0])) + fabsf(f2lo(x[1]))) + (fabsf(f2lo(x[2])) + fabsf(f2lo(x[3])));
+    hi = (fabsf(f2hi(x[0])) + fabsf(f2hi(x[1]))) + (fabsf(f2hi(x[2])) + fabsf(f2hi(x[3])));
+}
+
+__device__ __forceinline__ uint64_t clamp2(uint64_t v, float lim) {
+    return f2(fminf(fmaxf(f2lo(v), -lim), lim), fminf(fmaxf(f2hi(v), -lim), lim));
+}
+
+// Least-squares sums of the thread's columns: n_j += alpha_i z_ij X'_ij and
+// d_j += alpha_i z_ij^2 with z_ij = rne(X'_ij / c_j), clamped to +-qmax when
+// CLIP (App. C.1).
+template <int B, bool CLIP>
+__device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_t (&x2)[8][4],
+                                        const uint64_t (&g)[4], uint64_t (&n)[4], uint64_t (&d)[4]) {
+    constexpr float fqm = (float)((1 << (B - 1)) - 1);
+    const uint64_t M2 = f2s(kMagic), nM2 = f2s(-kMagic);
+#pragma unroll
+    for (int p = 0; p < 4; p++) {
+        uint64_t alo, ahi;
+        row_pairs(S.rAl, t, p, alo, ahi);
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+            const int m = 2 * p + h;
+            const uint64_t al = h ? ahi : alo;
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                uint64_t q = fadd2(fadd2(fmul2(x2[m][c], g[c]), M2), nM2);
+                if (CLIP) q = clamp2(q, fqm);
+                const uint64_t aq = fmul2(al, q);
+                n[c] = ffma2(aq, x2[m][c], n[c]);
+                d[c] = ffma2(aq, q, d[c]);
+            }
+        }
+    }
+}
+
+// Final codes q_ij = rne(X'_ij / c_j) with the stored scales (clamped when
+// CLIP), packed into the page chunks.
+template <int B, bool CLIP>
+__device__ __forceinline__ void final_codes(const T &t, const Smem &S, uint8_t *page,
+                                            const uint64_t (&x2)[8][4]) {
+    constexpr float fqm = (float)((1 << (B - 1)) - 1);
+    const uint64_t MB = f2s(kMagic + (float)(1 << (B - 1)));
+#pragma unroll
+    for (int c = 0; c < 4; c++) {
+        const uint64_t gc = col_pair(S.colG, t.col(c));
+        uint32_t f[16];
+#pragma unroll
+        for (int m = 0; m < 8; m++) {
+            uint64_t tq = fmul2(x2[m][c], gc);
+            if (CLIP) tq = clamp2(tq, fqm);
+            const uint64_t uu = fadd2(tq, MB);          // bits: 0x4B400000 | (q + 2^(B-1))
+            f[2 * m] = (uint32_t)uu;
+            f[2 * m + 1] = (uint32_t)(uu >> 32);
+        }
+        uint32_t wd[8];
+        pack_codes<B>(f, wd);
+        store_chunk<B>(page + chunk_off<B>(t.w, t.col(c)), wd);
+    }
 }
 
 // ---------------------------------------------------------------- the fit
 // Key-Row-Aware Dual-axis Fitting of the register tile (Sec. 4.3, App. C.1)
 // and packing into the page (App. C.3 step 6). The tile holds Z with
 // X_ij = a_i Z_ij (a_i > 0 a per-row factor: a_i = alpha r_i in the decode
-// step, 1 when packing a dense state); rs[r] holds the partial sums of |Z| of
-// the thread's rows over its 4 columns. Readout partials (y_part), when given,
-// ride on the column-start reduction round. On return the page holds r, c and
-// the codes. Requires the old page to be fully consumed by every thread.
+// step, 1 when packing a dense state, S.rA holds it when `scaled`); rs[r] holds
+// the partial sums of |Z| of the thread's rows over its 4 columns. Readout
+// partials (y_part), when given, ride on the column-start round and are summed
+// by warp w for columns 16w..16w+15. On return the page holds r, c and the
+// codes. Requires the old page to be fully consumed by every thread and
+// S.colM zeroed before the previous CTA barrier.
 template <int B>
 __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *page, const float *w2v,
-                                         const float *wisv, const float *a_row, uint64_t (&x2)[16][2],
+                                         const float *wisv, bool scaled, uint64_t (&x2)[8][4],
                                          float (&rs)[16], const float (&y_part)[4], bool with_y,
                                          float *y_out, int fit_iters) {
     constexpr int qm = (1 << (B - 1)) - 1;
@@ -242,102 +359,82 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         int rr;
         const float sz = warp_row_sums(rs, t.l, rr);
         const int i = t.row(rr);
-        const float a = a_row ? a_row[i] : 1.f;
+        const float a = scaled ? S.rA[i] : 1.f;
         const float m = (a * sz) * (1.0f / 128.0f);
         const float rf = __half2float(__float2half_rn(
             fminf(fmaxf(__fmul_rn(sqrtf(m), wisv[i]), kF16Min), kF16Max)));
         if ((t.l & 1) == 0) {
-            const float rho_a = __frcp_rn(rf) * a;                 // X' = rho_i X = (rho_i a_i) Z
-            const float al = w2v[i] * (rf * rf);                   // w_i^2 r_i^2
-            S.rowf[i] = make_float4(rho_a, rho_a, al, al);
+            S.rRho[i] = __frcp_rn(rf) * a;                 // X' = rho_i X = (rho_i a_i) Z
+            S.rAl[i] = w2v[i] * (rf * rf);                 // w_i^2 r_i^2
             page_r[i] = f16_bits(rf);
         }
     }
     __syncwarp();
-    // X' = X rho_i (row-normalised state) and the clip-free column start.
+    // X' = X rho_i (row-normalised state) and the clip-free column start,
+    // max_i |X'_ij| merged across warps by an atomic max on the (non-negative)
+    // float bits: exact and order-free.
     float cm[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int r = 0; r < 16; r++) {
-        const uint4 rf = *(const uint4 *)&S.rowf[t.row(r)];
-        const uint64_t rho = ((uint64_t)rf.y << 32) | rf.x;
-        x2[r][0] = fmul2(x2[r][0], rho);
-        x2[r][1] = fmul2(x2[r][1], rho);
-        cm[0] = fmaxf(cm[0], fabsf(f2lo(x2[r][0])));
-        cm[1] = fmaxf(cm[1], fabsf(f2hi(x2[r][0])));
-        cm[2] = fmaxf(cm[2], fabsf(f2lo(x2[r][1])));
-        cm[3] = fmaxf(cm[3], fabsf(f2hi(x2[r][1])));
-    }
-    {
-        float v[2][4];
+    for (int p = 0; p < 4; p++) {
+        uint64_t rlo, rhi;
+        row_pairs(S.rRho, t, p, rlo, rhi);
 #pragma unroll
         for (int c = 0; c < 4; c++) {
-            v[0][c] = cm[c];
-            v[1][c] = with_y ? y_part[c] : 0.f;
+            x2[2 * p][c] = fmul2(x2[2 * p][c], rlo);
+            x2[2 * p + 1][c] = fmul2(x2[2 * p + 1][c], rhi);
+            cm[c] = fmax3(cm[c], fabsf(f2lo(x2[2 * p][c])), fabsf(f2hi(x2[2 * p][c])));
+            cm[c] = fmax3(cm[c], fabsf(f2lo(x2[2 * p + 1][c])), fabsf(f2hi(x2[2 * p + 1][c])));
         }
-        cols_to_red<2>(t, S.red, v);
     }
-    if (t.tid == 0) {
-        S.flags[1] = 0;
-        S.flags[2] = 0;
+#pragma unroll
+    for (int c = 0; c < 4; c++) atomicMax(&S.colM[t.col(c)], __float_as_uint(cm[c]));
+    if (with_y) {
+        const float v[1][4] = {{y_part[0], y_part[1], y_part[2], y_part[3]}};
+        cols_to_red<1>(t, S.red, 2, v);
     }
+    if (t.tid == 0) S.flags[2] = 0;
     __syncthreads();
-    if (t.tid < 128) {
-        float mx = S.red[t.tid];
+    // Every thread derives the start of its own columns (identical in all warps).
+    uint64_t g[4];
+    bool capped = false;
 #pragma unroll
-        for (int wv = 1; wv < 8; wv++) mx = fmaxf(mx, S.red[wv * 128 + t.tid]);
+    for (int c = 0; c < 4; c++) {
+        const float mx = __uint_as_float(S.colM[t.col(c)]);
         const float c0 = __fmul_rn(mx, mu);
-        if (c0 > kF16Max) S.flags[1] = 1;                 // start capped: codes may clip
-        const float c = fminf(fmaxf(c0, kF16Min), kF16Max);
-        S.colC[t.tid] = c;
-        S.colG[pair_idx(t.tid)] = __frcp_rn(c);
-        S.colX[t.tid] = mx;                               // max_i |X'_ij|
-    } else if (with_y) {
-        const int j = t.tid - 128;
-        float s = S.red[8 * 128 + j];
+        capped |= c0 > kF16Max;                          // start capped: codes may clip
+        const float cc = fminf(fmaxf(c0, kF16Min), kF16Max);
+        const float gi = __frcp_rn(cc);
+        g[c] = f2(gi, gi);
+        if (t.w == 0) {
+            S.colC[t.col(c)] = cc;
+            S.colX[t.col(c)] = mx;
+        }
+    }
+    // every warp holds all 128 columns, so this is the same flag in every warp
+    const bool clip0 = __any_sync(0xffffffffu, capped);
+    if (with_y && t.l < 16) {
+        const int j = 16 * t.w + t.l;
+        float s = S.red[(2 * 8) * 128 + j];
 #pragma unroll
-        for (int wv = 1; wv < 8; wv++) s += S.red[(8 + wv) * 128 + j];
+        for (int wv = 1; wv < 8; wv++) s += S.red[(2 * 8 + wv) * 128 + j];
         y_out[j] = s;
     }
-    __syncthreads();
     // Fixed-code least-squares updates: c_j = sum alpha_i q_ij X'_ij / sum alpha_i q_ij^2
     // (alpha_i = w_i^2 r_i^2: the w^2-weighted objective in the X' domain).
-    const uint64_t M2 = f2s(kMagic), nM2 = f2s(-kMagic);
     for (int it = 0; it < fit_iters; it++) {
-        const bool clip = it > 0 || S.flags[1];
-        const uint64_t g01 = load_pair(S.colG, t.l, 0);
-        const uint64_t g23 = load_pair(S.colG, t.l, 1);
-        uint64_t n01 = 0, n23 = 0, d01 = 0, d23 = 0, e01 = 0, e23 = 0, h01 = 0, h23 = 0;
+        const bool clip = it > 0 || clip0;
+        if (it > 0) {
 #pragma unroll
-        for (int r = 0; r < 16; r++) {
-            const uint4 rf = *(const uint4 *)&S.rowf[t.row(r)];
-            const uint64_t al = ((uint64_t)rf.w << 32) | rf.z;
-            uint64_t q01 = fadd2(fadd2(fmul2(x2[r][0], g01), M2), nM2);
-            uint64_t q23 = fadd2(fadd2(fmul2(x2[r][1], g23), M2), nM2);
-            if (clip) {
-                q01 = f2(fminf(fmaxf(f2lo(q01), -fqm), fqm), fminf(fmaxf(f2hi(q01), -fqm), fqm));
-                q23 = f2(fminf(fmaxf(f2lo(q23), -fqm), fqm), fminf(fmaxf(f2hi(q23), -fqm), fqm));
-            }
-            const uint64_t a01 = fmul2(al, q01), a23 = fmul2(al, q23);
-            if (r & 1) {
-                e01 = ffma2(a01, x2[r][0], e01);
-                e23 = ffma2(a23, x2[r][1], e23);
-                h01 = ffma2(a01, q01, h01);
-                h23 = ffma2(a23, q23, h23);
-            } else {
-                n01 = ffma2(a01, x2[r][0], n01);
-                n23 = ffma2(a23, x2[r][1], n23);
-                d01 = ffma2(a01, q01, d01);
-                d23 = ffma2(a23, q23, d23);
-            }
+            for (int c = 0; c < 4; c++) g[c] = col_pair(S.colG, t.col(c));
         }
-        n01 = fadd2(n01, e01);
-        n23 = fadd2(n23, e23);
-        d01 = fadd2(d01, h01);
-        d23 = fadd2(d23, h23);
+        uint64_t n[4] = {0, 0, 0, 0}, d[4] = {0, 0, 0, 0};
+        // the clip decision is per tile: one branch here, none per element
+        if (clip) ls_sums<B, true>(t, S, x2, g, n, d);
+        else ls_sums<B, false>(t, S, x2, g, n, d);
         {
-            float v[2][4] = {{f2lo(n01), f2hi(n01), f2lo(n23), f2hi(n23)},
-                             {f2lo(d01), f2hi(d01), f2lo(d23), f2hi(d23)}};
-            cols_to_red<2>(t, S.red, v);
+            const float v[2][4] = {{pair_sum(n[0]), pair_sum(n[1]), pair_sum(n[2]), pair_sum(n[3])},
+                                   {pair_sum(d[0]), pair_sum(d[1]), pair_sum(d[2]), pair_sum(d[3])}};
+            cols_to_red<2>(t, S.red, 0, v);
         }
         __syncthreads();
         if (t.tid < 128) {
@@ -352,55 +449,36 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
             if (den > 0.f) c = fminf(fmaxf(__fdividef(num, den), kF16Min), kF16Max);
             if (it + 1 < fit_iters) {
                 S.colC[t.tid] = c;
-                S.colG[pair_idx(t.tid)] = __frcp_rn(c);
+                const float gi = __frcp_rn(c);
+                S.colG[t.tid] = make_float2(gi, gi);
             } else {
                 // storage precision of c; codes can clip only where max |X'| / c >= qmax + 1/2
                 const float cf = __half2float(__float2half_rn(c));
-                const float g = __frcp_rn(cf);
+                const float gi = __frcp_rn(cf);
                 page_c[t.tid] = f16_bits(cf);
-                S.colG[pair_idx(t.tid)] = g;
-                if (__fmul_rn(S.colX[t.tid], g) >= fqm + 0.5f) S.flags[2] = 1;
+                S.colG[t.tid] = make_float2(gi, gi);
+                if (__fmul_rn(S.colX[t.tid], gi) >= fqm + 0.5f) S.flags[2] = 1;
             }
         }
         __syncthreads();
     }
     // Final codes with the stored scales.
     const bool clip = S.flags[2] != 0;
-    const uint64_t MB = f2s(kMagic + (float)(1 << (B - 1)));
-#pragma unroll
-    for (int c = 0; c < 4; c += 2) {
-        const uint64_t g = load_pair(S.colG, t.l, c >> 1);
-        uint32_t ua[16], ub[16];
-#pragma unroll
-        for (int r = 0; r < 16; r++) {
-            uint64_t tq = fmul2(x2[r][c >> 1], g);
-            if (clip)
-                tq = f2(fminf(fmaxf(f2lo(tq), -fqm), fqm), fminf(fmaxf(f2hi(tq), -fqm), fqm));
-            const uint64_t uu = fadd2(tq, MB);              // bits: 0x4B400000 + (q + 2^(B-1))
-            ua[r] = (uint32_t)uu;
-            ub[r] = (uint32_t)(uu >> 32);
-        }
-        uint32_t wd[8];
-        pack16<B>(ua, wd);
-        store_chunk<B>(page + chunk_off<B>(t.w, t.col(c)), wd);
-        pack16<B>(ub, wd);
-        store_chunk<B>(page + chunk_off<B>(t.w, t.col(c + 1)), wd);
-    }
+    if (clip) final_codes<B, true>(t, S, page, x2);
+    else final_codes<B, false>(t, S, page, x2);
 }
 
-// FP16 pivot head: store fp16(a_i Z) (saturating) in band-major order.
-__device__ __forceinline__ void pack_pivot(const T &t, uint8_t *page, const uint64_t (&x2)[16][2],
+// FP16 pivot head: store fp16(a_i Z) (saturating) in band-major order; a row
+// pair is one 32-bit word of the chunk.
+__device__ __forceinline__ void pack_pivot(const T &t, uint8_t *page, const uint64_t (&x2)[8][4],
                                            float a) {
 #pragma unroll
     for (int c = 0; c < 4; c++) {
         uint32_t wd[8];
 #pragma unroll
-        for (int r = 0; r < 16; r += 2) {
-            const float za = (c & 1) ? f2hi(x2[r][c >> 1]) : f2lo(x2[r][c >> 1]);
-            const float zb = (c & 1) ? f2hi(x2[r + 1][c >> 1]) : f2lo(x2[r + 1][c >> 1]);
-            wd[r >> 1] = (uint32_t)f16_bits(f16_round_sat(a * za)) |
-                         ((uint32_t)f16_bits(f16_round_sat(a * zb)) << 16);
-        }
+        for (int m = 0; m < 8; m++)
+            wd[m] = (uint32_t)f16_bits(f16_round_sat(a * f2lo(x2[m][c]))) |
+                    ((uint32_t)f16_bits(f16_round_sat(a * f2hi(x2[m][c]))) << 16);
         store_chunk<kPivot>(page + chunk_off<kPivot>(t.w, t.col(c)), wd);
     }
 }
@@ -408,32 +486,26 @@ __device__ __forceinline__ void pack_pivot(const T &t, uint8_t *page, const uint
 // Reconstruct the column-scaled codes c_j q_ij (exact in fp32) or the FP16
 // values of a pivot head; the row factor stays separate.
 template <int B>
-__device__ __forceinline__ void load_tile(const T &t, const uint8_t *page, uint64_t (&x2)[16][2]) {
+__device__ __forceinline__ void load_tile(const T &t, const uint8_t *page, uint64_t (&x2)[8][4]) {
     const uint16_t *page_c = (const uint16_t *)(page + 256);
 #pragma unroll
-    for (int c = 0; c < 4; c += 2) {
-        uint32_t wa[8], wb[8];
-        load_chunk<B>(page + chunk_off<B>(t.w, t.col(c)), wa);
-        load_chunk<B>(page + chunk_off<B>(t.w, t.col(c + 1)), wb);
+    for (int c = 0; c < 4; c++) {
+        uint32_t wd[8];
+        load_chunk<B>(page + chunk_off<B>(t.w, t.col(c)), wd);
         if (B == kPivot) {
 #pragma unroll
-            for (int r = 0; r < 16; r++) {
-                const float a = f16_val((uint16_t)(wa[r >> 1] >> (16 * (r & 1))));
-                const float b = f16_val((uint16_t)(wb[r >> 1] >> (16 * (r & 1))));
-                x2[r][c >> 1] = f2(a, b);
-            }
+            for (int m = 0; m < 8; m++)
+                x2[m][c] = f2(f16_val((uint16_t)(wd[m] & 0xFFFFu)), f16_val((uint16_t)(wd[m] >> 16)));
         } else {
-            const float ca = f16_val(page_c[t.col(c)]), cb = f16_val(page_c[t.col(c + 1)]);
-            // 0x4B400000 + u - 2^(B-1) is the float 1.5*2^23 + q; fma(f, c, -1.5*2^23 c)
-            // = c q exactly (c fp16, |q| <= 127: 19 significant bits; 1.5*2^23 c exact).
-            constexpr uint32_t kBias = 0x4B400000u - (1u << (B - 1));
-            const uint64_t cc = f2(ca, cb), oc = f2(-kMagic * ca, -kMagic * cb);
+            // f = 1.5*2^23 + u s (s = 1 or the pair's high scale): fma(f, c/s, -1.5*2^23 c/s)
+            // = c u exactly (c fp16 and normal, u < 2^8: 19 significant bits; the
+            // offset has 12), and c u - c 2^(B-1) = c q is exact as well.
+            const float cj = f16_val(page_c[t.col(c)]);
+            constexpr float hs = hi_scale<B>();
+            const uint64_t cc = f2(cj, cj * hs), oc = f2(-kMagic * cj, (-kMagic * cj) * hs);
+            const uint64_t bc = f2s(-(float)(1 << (B - 1)) * cj);
 #pragma unroll
-            for (int r = 0; r < 16; r++) {
-                const uint64_t fq = ((uint64_t)(code_at<B>(wb, r) + kBias) << 32) |
-                                    (uint64_t)(code_at<B>(wa, r) + kBias);
-                x2[r][c >> 1] = ffma2(fq, cc, oc);
-            }
+            for (int m = 0; m < 8; m++) x2[m][c] = fadd2(ffma2(code_pair<B>(wd, m), cc, oc), bc);
         }
     }
 }
@@ -444,7 +516,7 @@ struct DecodeArgs {
     uint64_t stride;
     int pool_slots;
     const int32_t *slots;
-    int Hk, Hv, items;
+    int Hk, Hv, nb, items;     // nb batch entries; item = head * nb + entry
     LayerTables tab;
     const float *q, *k, *v, *beta, *gate;
     float *y;
@@ -458,10 +530,9 @@ __device__ __forceinline__ bool slot_ok(const DecodeArgs &a, int slot) {
     return slot >= 0 && slot < a.pool_slots;
 }
 
-// Producer: start the copies of `item` (batch entry b = item / Hv, head h) into
-// stage s (thread 0 only). An invalid slot completes the phase without data.
-__device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int item, int slot, int s) {
-    const int b = item / a.Hv, h = item - b * a.Hv;
+// Producer: start the copies of the item (head h, batch entry b) into stage s
+// (one thread). An invalid slot completes the phase without data.
+__device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s) {
     uint64_t *bar = &S.bars[s];
     if (!slot_ok(a, slot)) {
         mbar_arrive(bar);
@@ -469,7 +540,7 @@ __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int it
     }
     Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
     const uint32_t nb = S.hbytes[h];
-    const int hk = h / (a.Hv / a.Hk);
+    const int hk = S.hkey[h];
     mbar_arrive_tx(bar, nb + kVecBytes);
     bulk_load(st.page, a.pool + (uint64_t)slot * a.stride + S.hoff[h], nb, bar);
     bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
@@ -480,154 +551,199 @@ __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int it
 }
 
 // One decode step of one head page staged in shared memory (width B).
-// `refill` runs once the stage's inputs are fully consumed (after the retrieval
-// reduction); the page itself is rewritten in place afterwards.
+// `ok` is this thread's verdict on the stage's copies; the first CTA barrier
+// takes the OR of the negations, and on a stalled copy every thread returns
+// false there (what it read before is discarded). `refill` runs after that
+// barrier; the page itself is rewritten in place afterwards.
 //
 // With a_i = alpha r_i (> 0) and Z_ij = c_j q_ij + (beta k_i / a_i) delta_j the
 // update is X_ij = a_i Z_ij: one fma per element instead of two.
 template <int B, class Refill>
-__device__ __forceinline__ void decode_item(const T &t, const Smem &S, const Stage &st, float alpha,
-                                            float beta, float *y_out, int fit_iters,
+__device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Stage &st, float alpha,
+                                            float beta, float *y_out, int fit_iters, bool ok,
                                             const Refill &refill) {
     const uint16_t *page_r = (const uint16_t *)st.page;
-    // Row constants of the warp's band (warp-local): a_i, kappa_i = k_i a_i,
-    // beta k_i / a_i, q_i a_i, as duplicated fp32 pairs.
+    // Row constants of the warp's band (warp-local).
     if (t.l < 16) {
         const int i = t.row(t.l);
         const float a = fmaxf(B == kPivot ? alpha : alpha * f16_val(page_r[i]), 1e-30f);
         const float ki = st.k[i];
-        const float kap = ki * a, bkp = __fdiv_rn(beta * ki, a), qa = st.q[i] * a;
-        S.rowc[2 * i] = make_float4(kap, kap, bkp, bkp);
-        S.rowc[2 * i + 1] = make_float4(qa, qa, a, a);
-        S.rowa[i] = a;
+        S.rKap[i] = ki * a;
+        S.rBkp[i] = __fdividef(beta * ki, a);          // within 2 ulp: Z carries rounding anyway
+        S.rQa[i] = st.q[i] * a;
+        S.rA[i] = a;
     }
-    uint64_t x2[16][2];
+    if (t.tid < 128) S.colM[t.tid] = 0u;
+    uint64_t x2[8][4];
     load_tile<B>(t, st.page, x2);
     __syncwarp();
     // Step 2a: retrieval u_j = sum_i k_i a_i (c_j q_ij).
-    uint64_t u01 = 0, u23 = 0, v01 = 0, v23 = 0;
-#pragma unroll
-    for (int r = 0; r < 16; r++) {
-        const uint4 rc = *(const uint4 *)&S.rowc[2 * t.row(r)];
-        const uint64_t kap = ((uint64_t)rc.y << 32) | rc.x;
-        if (r & 1) {
-            v01 = ffma2(kap, x2[r][0], v01);
-            v23 = ffma2(kap, x2[r][1], v23);
-        } else {
-            u01 = ffma2(kap, x2[r][0], u01);
-            u23 = ffma2(kap, x2[r][1], u23);
-        }
-    }
-    u01 = fadd2(u01, v01);
-    u23 = fadd2(u23, v23);
     {
-        float v[1][4] = {{f2lo(u01), f2hi(u01), f2lo(u23), f2hi(u23)}};
-        cols_to_red<1>(t, S.red, v);
+        uint64_t ua[4] = {0, 0, 0, 0}, ub[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int p = 0; p < 4; p++) {
+            uint64_t klo, khi;
+            row_pairs(S.rKap, t, p, klo, khi);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                ua[c] = ffma2(klo, x2[2 * p][c], ua[c]);
+                ub[c] = ffma2(khi, x2[2 * p + 1][c], ub[c]);
+            }
+        }
+        const float v[1][4] = {{pair_sum(fadd2(ua[0], ub[0])), pair_sum(fadd2(ua[1], ub[1])),
+                                pair_sum(fadd2(ua[2], ub[2])), pair_sum(fadd2(ua[3], ub[3]))}};
+        cols_to_red<1>(t, S.red, 0, v);
     }
-    __syncthreads();
+    if (__syncthreads_or(!ok)) return false;
     if (t.tid < 128) {
         float s = 0.f;
 #pragma unroll
         for (int wv = 0; wv < 8; wv++) s += S.red[wv * 128 + t.tid];
-        S.colD[pair_idx(t.tid)] = st.v[t.tid] - s;          // delta_j = v_j - u_j
+        const float dl = st.v[t.tid] - s;                  // delta_j = v_j - u_j
+        S.colD[t.tid] = make_float2(dl, dl);
     }
     refill();
     __syncthreads();
     // Step 2b-3: Z = c q + (beta k / a) delta; readout partials q_i a_i Z_ij.
-    const uint64_t dl01 = load_pair(S.colD, t.l, 0);
-    const uint64_t dl23 = load_pair(S.colD, t.l, 1);
-    uint64_t y01 = 0, y23 = 0, z01 = 0, z23 = 0;
+    uint64_t dl[4];
+#pragma unroll
+    for (int c = 0; c < 4; c++) dl[c] = col_pair(S.colD, t.col(c));
+    uint64_t ya[4] = {0, 0, 0, 0}, yb[4] = {0, 0, 0, 0};
     float rs[16];
 #pragma unroll
-    for (int r = 0; r < 16; r++) {
-        const uint4 rc = *(const uint4 *)&S.rowc[2 * t.row(r)];
-        const uint4 rq = *(const uint4 *)&S.rowc[2 * t.row(r) + 1];
-        const uint64_t bkp = ((uint64_t)rc.w << 32) | rc.z;
-        const uint64_t qa = ((uint64_t)rq.y << 32) | rq.x;
-        x2[r][0] = ffma2(bkp, dl01, x2[r][0]);
-        x2[r][1] = ffma2(bkp, dl23, x2[r][1]);
-        if (r & 1) {
-            z01 = ffma2(qa, x2[r][0], z01);
-            z23 = ffma2(qa, x2[r][1], z23);
-        } else {
-            y01 = ffma2(qa, x2[r][0], y01);
-            y23 = ffma2(qa, x2[r][1], y23);
-        }
-        rs[r] = (fabsf(f2lo(x2[r][0])) + fabsf(f2hi(x2[r][0]))) +
-                (fabsf(f2lo(x2[r][1])) + fabsf(f2hi(x2[r][1])));
-    }
-    y01 = fadd2(y01, z01);
-    y23 = fadd2(y23, z23);
-    const float yp[4] = {f2lo(y01), f2hi(y01), f2lo(y23), f2hi(y23)};
-    if (B == kPivot) {
-        float v[1][4] = {{yp[0], yp[1], yp[2], yp[3]}};
-        cols_to_red<1>(t, S.red, v);
-        __syncthreads();
-        if (t.tid < 128) {
-            float s = 0.f;
+    for (int p = 0; p < 4; p++) {
+        uint64_t blo, bhi, qlo, qhi;
+        row_pairs(S.rBkp, t, p, blo, bhi);
+        row_pairs(S.rQa, t, p, qlo, qhi);
 #pragma unroll
-            for (int wv = 0; wv < 8; wv++) s += S.red[wv * 128 + t.tid];
-            y_out[t.tid] = s;
+        for (int c = 0; c < 4; c++) {
+            x2[2 * p][c] = ffma2(blo, dl[c], x2[2 * p][c]);
+            x2[2 * p + 1][c] = ffma2(bhi, dl[c], x2[2 * p + 1][c]);
+            ya[c] = ffma2(qlo, x2[2 * p][c], ya[c]);
+            yb[c] = ffma2(qhi, x2[2 * p + 1][c], yb[c]);
+        }
+        abs_row_sums(x2[2 * p], rs[4 * p], rs[4 * p + 1]);
+        abs_row_sums(x2[2 * p + 1], rs[4 * p + 2], rs[4 * p + 3]);
+    }
+    const float yp[4] = {pair_sum(fadd2(ya[0], yb[0])), pair_sum(fadd2(ya[1], yb[1])),
+                         pair_sum(fadd2(ya[2], yb[2])), pair_sum(fadd2(ya[3], yb[3]))};
+    if (B == kPivot) {
+        const float v[1][4] = {{yp[0], yp[1], yp[2], yp[3]}};
+        cols_to_red<1>(t, S.red, 2, v);
+        __syncthreads();
+        if (t.l < 16) {
+            const int j = 16 * t.w + t.l;
+            float s = S.red[(2 * 8) * 128 + j];
+#pragma unroll
+            for (int wv = 1; wv < 8; wv++) s += S.red[(2 * 8 + wv) * 128 + j];
+            y_out[j] = s;
         }
         pack_pivot(t, st.page, x2, fmaxf(alpha, 1e-30f));
-        return;
+        return true;
     }
     // Steps 4-6: refit and repack in place.
-    fit_pack<B>(t, S, st.page, st.w2, st.wis, S.rowa, x2, rs, yp, true, y_out, fit_iters);
+    fit_pack<B>(t, S, st.page, st.w2, st.wis, true, x2, rs, yp, true, y_out, fit_iters);
+    return true;
 }
+
+// (head, batch entry) of item = head * nb + entry, stepped by the grid stride
+// G = gq * nb + gr without divisions.
+struct Cursor {
+    int item, h, b;
+    __device__ __forceinline__ Cursor(int it, int nb) : item(it), h(it / nb), b(it - (it / nb) * nb) {}
+    __device__ __forceinline__ void step(int G, int gq, int gr, int nb) {
+        item += G;
+        h += gq;
+        b += gr;
+        if (b >= nb) {
+            b -= nb;
+            h++;
+        }
+    }
+};
 
 __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     const T t;
     const Smem S(smem);
     const int G = gridDim.x, S_n = a.n_stages;
+    const int gq = G / a.nb, gr = G - gq * a.nb;
     const int first = blockIdx.x;
     if (first >= a.items) return;
+    const int grp = a.Hv / a.Hk;
     for (int h = t.tid; h < a.Hv; h += kThreads) {
         S.hoff[h] = a.tab.head_off[h];
         S.hbytes[h] = a.tab.head_bytes[h];
         S.hbits[h] = a.tab.head_bits[h];
+        S.hkey[h] = (uint8_t)(h / grp);
     }
     if (t.tid == kProducer) {
         for (int s = 0; s < S_n; s++) mbar_init(&S.bars[s], 1);
         mbar_init_fence();
     }
     __syncthreads();
-    if (t.tid == kProducer) {
-        for (int s = 0; s < S_n; s++) {
-            const int item = first + s * G;
-            if (item < a.items) issue(a, S, item, a.slots[item / a.Hv], s);
-        }
-    }
     // With three or more stages a stage is refilled two items after its own item
     // (its store has long finished reading it); with two stages, one item after.
     const int lag = S_n >= 3 ? 2 : 1;
-    // scalars of the current item; the next item's are fetched one iteration ahead
-    int b = first / a.Hv, h = first - b * a.Hv;
-    int slot = a.slots[b];
-    float alpha = a.gate[(size_t)b * a.Hv + h], beta = a.beta[(size_t)b * a.Hv + h];
-    int n = 0;
-    for (int item = first; item < a.items; item += G, n++) {
-        const int s = n % S_n;
-        const uint32_t parity = (uint32_t)(n / S_n) & 1u;
-        // prefetch: next item's scalars (all threads), and the slot of the item
-        // this iteration will issue (thread 0)
-        const int nitem = item + G;
-        int nb = 0, nh = 0, nslot = -1;
-        float nalpha = 0.f, nbeta = 0.f;
-        if (nitem < a.items) {
-            nb = nitem / a.Hv;
-            nh = nitem - nb * a.Hv;
-            nslot = a.slots[nb];
-            nalpha = a.gate[(size_t)nb * a.Hv + nh];
-            nbeta = a.beta[(size_t)nb * a.Hv + nh];
+    if (t.tid == kProducer) {
+        Cursor c0(first, a.nb);
+        for (int s = 0; s < S_n && c0.item < a.items; s++) {
+            issue(a, S, c0.h, c0.b, a.slots[c0.b], s);
+            c0.step(G, gq, gr, a.nb);
         }
-        const int iitem = first + (n - lag + S_n) * G;
+    }
+    // iteration n >= lag refills stage (n - lag) mod S with item n - lag + S
+    Cursor cur(first, a.nb), iss(first + S_n * G, a.nb);
+    // scalars of the current item; the next item's are fetched one iteration ahead
+    int slot = a.slots[cur.b];
+    float alpha = a.gate[(size_t)cur.b * a.Hv + cur.h], beta = a.beta[(size_t)cur.b * a.Hv + cur.h];
+    int s = 0, is = 0;                    // stage of the current item, stage refilled next
+    uint32_t parity = 0;
+    for (int n = 0; cur.item < a.items; n++) {
+        // prefetch: next item's scalars (all threads), and the slot of the item
+        // this iteration will issue (producer)
+        Cursor nxt = cur;
+        nxt.step(G, gq, gr, a.nb);
+        int nslot = -1;
+        float nalpha = 0.f, nbeta = 0.f;
+        if (nxt.item < a.items) {
+            nslot = a.slots[nxt.b];
+            nalpha = a.gate[(size_t)nxt.b * a.Hv + nxt.h];
+            nbeta = a.beta[(size_t)nxt.b * a.Hv + nxt.h];
+        }
+        const bool do_issue = n >= lag && iss.item < a.items;
         int islot = -1;
-        if (t.tid == kProducer && n >= lag && iitem < a.items) islot = a.slots[iitem / a.Hv];
+        if (t.tid == kProducer && do_issue) islot = a.slots[iss.b];
 
         const bool ok = mbar_wait(&S.bars[s], parity, kWaitCycles);
-        if (__syncthreads_or(!ok)) {
+        const bool valid = slot_ok(a, slot);
+        if (!valid && t.tid == 0) raise_error(a.err, STEPQ_ERR_SLOT_RANGE);
+        const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
+        // Refill the stage of an earlier item (its store was committed `lag`
+        // items ago) with the item S-1 ahead of it: S-1 items stay in flight.
+        const auto refill = [&]() {
+            if (t.tid == kProducer && do_issue) {
+                if (lag == 2) bulk_wait_read_all_but_one();
+                else bulk_wait_read_all();
+                issue(a, S, iss.h, iss.b, islot, is);
+            }
+        };
+        bool alive = true;
+        const int h = cur.h;
+        if (valid) {
+            float *y_out = a.y + ((size_t)cur.b * a.Hv + h) * 128;
+            switch (S.hbits[h]) {
+            case 2: alive = decode_item<2>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
+            case 4: alive = decode_item<4>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
+            case 6: alive = decode_item<6>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
+            case 8: alive = decode_item<8>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
+            default: alive = decode_item<kPivot>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
+            }
+        } else {
+            alive = !__syncthreads_or(!ok);
+            if (alive) refill();
+        }
+        if (!alive) {
             if (t.tid == kProducer) {
                 raise_error(a.err, STEPQ_ERR_TIMEOUT);
                 // drain this CTA's copies still in flight (items n .. issued), with a bound
@@ -640,30 +756,6 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
             }
             return;
         }
-        const bool valid = slot_ok(a, slot);
-        if (!valid && t.tid == 0) raise_error(a.err, STEPQ_ERR_SLOT_RANGE);
-        const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
-        // Refill the stage of the previous item (its store was committed one item
-        // ago) with the item S-1 ahead of it: S-1 items stay in flight.
-        const auto refill = [&]() {
-            if (t.tid == kProducer && n >= lag && iitem < a.items) {
-                if (lag == 2) bulk_wait_read_all_but_one();
-                else bulk_wait_read_all();
-                issue(a, S, iitem, islot, (n - lag) % S_n);
-            }
-        };
-        if (valid) {
-            float *y_out = a.y + ((size_t)b * a.Hv + h) * 128;
-            switch (S.hbits[h]) {
-            case 2: decode_item<2>(t, S, st, alpha, beta, y_out, a.fit_iters, refill); break;
-            case 4: decode_item<4>(t, S, st, alpha, beta, y_out, a.fit_iters, refill); break;
-            case 6: decode_item<6>(t, S, st, alpha, beta, y_out, a.fit_iters, refill); break;
-            case 8: decode_item<8>(t, S, st, alpha, beta, y_out, a.fit_iters, refill); break;
-            default: decode_item<kPivot>(t, S, st, alpha, beta, y_out, a.fit_iters, refill); break;
-            }
-        } else {
-            refill();
-        }
         __syncthreads();                                 // the page in stage s is final
         if (t.tid == kProducer) {
             if (valid) {
@@ -672,7 +764,16 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
             }
             bulk_commit();
         }
-        b = nb; h = nh; slot = nslot; alpha = nalpha; beta = nbeta;
+        cur = nxt;
+        slot = nslot; alpha = nalpha; beta = nbeta;
+        if (n >= lag) {
+            iss.step(G, gq, gr, a.nb);
+            if (++is == S_n) is = 0;
+        }
+        if (++s == S_n) {
+            s = 0;
+            parity ^= 1u;
+        }
     }
     if (t.tid == kProducer) bulk_wait_all();
 }
@@ -697,22 +798,21 @@ constexpr int kPoolSmem = kOffStages + kPageMaxHead + kVecBytes;
 template <int B>
 __device__ __forceinline__ void quantize_item(const T &t, const Smem &S, uint8_t *page, const float *w2,
                                               const float *wis, const float *X, int fit_iters) {
-    uint64_t x2[16][2];
+    uint64_t x2[8][4];
     float rs[16];
 #pragma unroll
-    for (int r = 0; r < 16; r++) {
-        const float *row = X + t.row(r) * 128;
-        const float a = row[t.col(0)], b = row[t.col(1)], c = row[t.col(2)], d = row[t.col(3)];
-        x2[r][0] = f2(a, b);
-        x2[r][1] = f2(c, d);
-        rs[r] = fabsf(a) + fabsf(b) + fabsf(c) + fabsf(d);
+    for (int m = 0; m < 8; m++) {
+        const float *r0 = X + t.row(2 * m) * 128, *r1 = r0 + 128;
+#pragma unroll
+        for (int c = 0; c < 4; c++) x2[m][c] = f2(r0[t.col(c)], r1[t.col(c)]);
+        abs_row_sums(x2[m], rs[2 * m], rs[2 * m + 1]);
     }
     if (B == kPivot) {
         pack_pivot(t, page, x2, 1.f);
         return;
     }
     const float none[4] = {0.f, 0.f, 0.f, 0.f};
-    fit_pack<B>(t, S, page, w2, wis, nullptr, x2, rs, none, false, nullptr, fit_iters);
+    fit_pack<B>(t, S, page, w2, wis, false, x2, rs, none, false, nullptr, fit_iters);
 }
 
 __global__ void __launch_bounds__(kThreads, 2) quantize_heads_kernel(PoolArgs a) {
@@ -730,8 +830,8 @@ __global__ void __launch_bounds__(kThreads, 2) quantize_heads_kernel(PoolArgs a)
     if (t.tid < 128) {
         w2[t.tid] = a.tab.w2[h * 128 + t.tid];
         wis[t.tid] = a.tab.wis[h * 128 + t.tid];
+        S.colM[t.tid] = 0u;
     }
-    if (t.tid == 0) S.flags[1] = 0;
     __syncthreads();
     const float *X = a.states + (size_t)b * a.state_stride_b + (size_t)h * kN;
     switch (a.tab.head_bits[h]) {
@@ -749,23 +849,19 @@ __global__ void __launch_bounds__(kThreads, 2) quantize_heads_kernel(PoolArgs a)
 
 template <int B>
 __device__ __forceinline__ void dequantize_item(const T &t, const uint8_t *page, float *out) {
-    uint64_t x2[16][2];
-    load_tile<B>(t, page, x2);      // c_j q_ij (rounded once) or the FP16 value
+    uint64_t x2[8][4];
+    load_tile<B>(t, page, x2);      // c_j q_ij (exact) or the FP16 value
     const uint16_t *page_r = (const uint16_t *)page;
 #pragma unroll
-    for (int r = 0; r < 16; r++) {
-        float *row = out + t.row(r) * 128;
+    for (int m = 0; m < 8; m++) {
+        float *r0 = out + t.row(2 * m) * 128, *r1 = r0 + 128;
+        // r_i c_j z_ij rounded once: c_j q_ij is exact in fp32 (fp16 x 8 bits)
+        const uint64_t rr = B == kPivot ? 0 : f2(f16_val(page_r[t.row(2 * m)]), f16_val(page_r[t.row(2 * m + 1)]));
 #pragma unroll
         for (int c = 0; c < 4; c++) {
-            float v;
-            if (B == kPivot) {
-                v = (c & 1) ? f2hi(x2[r][c >> 1]) : f2lo(x2[r][c >> 1]);
-            } else {
-                // r_i c_j z_ij rounded once: c_j q_ij is exact in fp32 (fp16 x 8 bits)
-                const float cq = (c & 1) ? f2hi(x2[r][c >> 1]) : f2lo(x2[r][c >> 1]);
-                v = __fmul_rn(f16_val(page_r[t.row(r)]), cq);
-            }
-            row[t.col(c)] = v;
+            const uint64_t v = B == kPivot ? x2[m][c] : fmul2(rr, x2[m][c]);
+            r0[t.col(c)] = f2lo(v);
+            r1[t.col(c)] = f2hi(v);
         }
     }
 }
@@ -829,6 +925,7 @@ stepq_status launch_decode_heads(const stepq_plan *p, int layer, uint8_t *pool, 
     a.slots = slots;
     a.Hk = p->cfg.n_key_heads;
     a.Hv = Hv;
+    a.nb = B;
     a.items = B * Hv;
     a.tab = p->layer(layer);
     a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
