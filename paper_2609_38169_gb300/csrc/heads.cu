@@ -341,7 +341,7 @@ __device__ __forceinline__ void final_codes(const T &t, const Smem &S, uint8_t *
 // step, 1 when packing a dense state, S.rA holds it when `scaled`); rs[r] holds
 // the partial sums of |Z| of the thread's rows over its 4 columns. Readout
 // partials (y_part), when given, ride on the column-start round and are summed
-// by warp w for columns 16w..16w+15. On return the page holds r, c and the
+// by threads 128..255 while threads 0..127 derive the start. On return the page holds r, c and the
 // codes. Requires the old page to be fully consumed by every thread and
 // S.colM zeroed before the previous CTA barrier.
 template <int B>
@@ -392,33 +392,34 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         const float v[1][4] = {{y_part[0], y_part[1], y_part[2], y_part[3]}};
         cols_to_red<1>(t, S.red, 2, v);
     }
-    if (t.tid == 0) S.flags[2] = 0;
+    if (t.tid == 0) {
+        S.flags[1] = 0;
+        S.flags[2] = 0;
+    }
     __syncthreads();
-    // Every thread derives the start of its own columns (identical in all warps).
-    uint64_t g[4];
-    bool capped = false;
-#pragma unroll
-    for (int c = 0; c < 4; c++) {
-        const float mx = __uint_as_float(S.colM[t.col(c)]);
+    // Column start (threads 0..127, one column each) beside the readout sums
+    // (threads 128..255).
+    if (t.tid < 128) {
+        const float mx = __uint_as_float(S.colM[t.tid]);
         const float c0 = __fmul_rn(mx, mu);
-        capped |= c0 > kF16Max;                          // start capped: codes may clip
+        if (c0 > kF16Max) S.flags[1] = 1;                 // start capped: codes may clip
         const float cc = fminf(fmaxf(c0, kF16Min), kF16Max);
         const float gi = __frcp_rn(cc);
-        g[c] = f2(gi, gi);
-        if (t.w == 0) {
-            S.colC[t.col(c)] = cc;
-            S.colX[t.col(c)] = mx;
-        }
-    }
-    // every warp holds all 128 columns, so this is the same flag in every warp
-    const bool clip0 = __any_sync(0xffffffffu, capped);
-    if (with_y && t.l < 16) {
-        const int j = 16 * t.w + t.l;
+        S.colC[t.tid] = cc;
+        S.colX[t.tid] = mx;
+        S.colG[t.tid] = make_float2(gi, gi);
+    } else if (with_y) {
+        const int j = t.tid - 128;
         float s = S.red[(2 * 8) * 128 + j];
 #pragma unroll
         for (int wv = 1; wv < 8; wv++) s += S.red[(2 * 8 + wv) * 128 + j];
         y_out[j] = s;
     }
+    __syncthreads();
+    const bool clip0 = S.flags[1] != 0;
+    uint64_t g[4];
+#pragma unroll
+    for (int c = 0; c < 4; c++) g[c] = col_pair(S.colG, t.col(c));
     // Fixed-code least-squares updates: c_j = sum alpha_i q_ij X'_ij / sum alpha_i q_ij^2
     // (alpha_i = w_i^2 r_i^2: the w^2-weighted objective in the X' domain).
     for (int it = 0; it < fit_iters; it++) {
@@ -500,10 +501,10 @@ __device__ __forceinline__ void load_tile(const T &t, const uint8_t *page, uint6
             // f = 1.5*2^23 + u s (s = 1 or the pair's high scale): fma(f, c/s, -1.5*2^23 c/s)
             // = c u exactly (c fp16 and normal, u < 2^8: 19 significant bits; the
             // offset has 12), and c u - c 2^(B-1) = c q is exact as well.
-            const float cj = f16_val(page_c[t.col(c)]);
-            constexpr float hs = hi_scale<B>();
-            const uint64_t cc = f2(cj, cj * hs), oc = f2(-kMagic * cj, (-kMagic * cj) * hs);
-            const uint64_t bc = f2s(-(float)(1 << (B - 1)) * cj);
+            const uint64_t cj = f2s(f16_val(page_c[t.col(c)]));
+            const uint64_t cc = fmul2(cj, f2(1.0f, hi_scale<B>()));
+            const uint64_t oc = fmul2(cc, f2s(-kMagic));
+            const uint64_t bc = fmul2(cj, f2s(-(float)(1 << (B - 1))));
 #pragma unroll
             for (int m = 0; m < 8; m++) x2[m][c] = fadd2(ffma2(code_pair<B>(wd, m), cc, oc), bc);
         }
