@@ -113,3 +113,13 @@ def test_host_only_plan_refuses_device_calls(oracle):
     fake = C.c_void_p(1 << 20)   # aligned, never dereferenced: the call must refuse first
     r = L.stepq_decode_step(plan.handle, 0, fake, 1, fake, 1, fake, fake, fake, fake, fake, fake, None)
     assert r == 5                                                             # STEPQ_ERR_CUDA
+
+
+def test_drift_variants_and_cli():
+    """The drift module's variant table and command line (no device work)."""
+    from paper_2609_38169_gb300 import drift
+    assert set(drift.VARIANTS) == {"stepq6", "stepq4", "int8", "int4"}
+    assert drift.VARIANTS["stepq4"]["candidates"] == (2, 4, 6, 8)
+    with pytest.raises(SystemExit) as e:
+        drift.main(["--help"])
+    assert e.value.code == 0
