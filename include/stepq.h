@@ -237,6 +237,10 @@ stepq_status stepq_validate_slots_noalloc(const int32_t *slots, int B, int pool_
 /* Read and clear the sticky device error of the current device (synchronises
  * `stream`): STEPQ_OK, or the first error a kernel raised. */
 stepq_status stepq_device_error(stepq_stream_t stream);
+/* The same read-and-clear of the sticky device error, under the name used for
+ * it in the boundary's design table: surfaces what the asynchronous calls queued
+ * on `stream` reported. Synchronises `stream`. */
+stepq_status stepq_stream_status(stepq_stream_t stream);
 
 const char *stepq_status_str(stepq_status s);
 const char *stepq_version(void);

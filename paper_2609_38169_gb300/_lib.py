@@ -50,6 +50,7 @@ SIGNATURES = {
     "stepq_validate_slots": (I, [P, I, I, P, P, P]),
     "stepq_validate_slots_noalloc": (I, [P, I, I, P, P]),
     "stepq_device_error": (I, [P]),
+    "stepq_stream_status": (I, [P]),
     "stepq_status_str": (C.c_char_p, [I]),
     "stepq_version": (C.c_char_p, []),
 }

@@ -316,6 +316,10 @@ def stepq_device_error(stream=None) -> int:
     return int(_lib.lib().stepq_device_error(_stream(stream)))
 
 
+def stepq_stream_status(stream=None) -> int:
+    return int(_lib.lib().stepq_stream_status(_stream(stream)))
+
+
 # ------------------------------------------------------------------ calibration driver
 @dataclass
 class CalibStats:

@@ -1,6 +1,6 @@
 // C-ABI entry points of the device path: argument checks, then one launch.
-// No entry point here synchronises or allocates except stepq_device_error(),
-// which reads the sticky device error.
+// No entry point here synchronises or allocates except stepq_device_error() and
+// stepq_stream_status(), which read the sticky device error.
 #include <cstdint>
 
 #include "internal.h"
@@ -205,6 +205,10 @@ extern "C" stepq_status stepq_validate_slots_noalloc(const int32_t *slots, int B
 }
 
 extern "C" stepq_status stepq_device_error(stepq_stream_t stream) {
+    return read_device_error((cudaStream_t)stream);
+}
+
+extern "C" stepq_status stepq_stream_status(stepq_stream_t stream) {
     return read_device_error((cudaStream_t)stream);
 }
 

@@ -199,6 +199,9 @@ def test_empty_batch_and_bad_slots(torch):
     A.stepq_decode_step(plan, 0, pool_d, bad, q, q, v, beta, gate, y, pool_slots=4)
     assert A.stepq_device_error() == 2                                          # STEPQ_ERR_SLOT_RANGE
     assert A.stepq_device_error() == 0                                          # cleared
+    A.stepq_decode_step(plan, 0, pool_d, bad, q, q, v, beta, gate, y, pool_slots=4)
+    assert A.stepq_stream_status() == 2                                         # same word, other name
+    assert A.stepq_stream_status() == 0
     assert torch.equal(pool_d, before)
     with pytest.raises(A._lib.StepqError):
         A.stepq_decode_step(plan, 1, pool_d, bad, q, q, v, beta, gate, y)       # layer out of range
