@@ -21,13 +21,12 @@
 #include "async.cuh"
 #include "device.cuh"
 #include "internal.h"
+#include "pipeline.cuh"
+#include "tile.cuh"
 
 namespace stepq {
 namespace hk {
 
-constexpr long long kWaitCycles = 2000000000LL;      // ~1 s at 2 GHz
-constexpr float kMagic = 12582912.0f;                  // 1.5 * 2^23: rint by addition
-constexpr uint32_t kMagicBits = 0x4B400000u;           // its bit pattern (low 22 bits zero)
 constexpr int kVecBytes = 5 * 512;                     // q k v w2 wis per stage
 
 // ------------------------------------------------------------ shared layout
@@ -92,8 +91,6 @@ struct Stage {
         wis = q + 512;
     }
 };
-
-constexpr int kProducer = kThreads - 32;              // lane 0 of the last warp issues copies
 
 struct T {   // thread coordinates
     int tid, w, l;
@@ -228,37 +225,6 @@ __device__ __forceinline__ void pack_codes(const uint32_t (&f)[16], uint32_t (&w
     for (int k = 0; k < NW; k++) wd[k] = acc[k];
 }
 
-// Sum of 16 per-row partials over the 32 lanes of a warp (reduce-scatter): lane
-// l returns the full sum of row 8*b4 + 4*b3 + 2*b2 + b1 (b_k = bit k of l).
-__device__ __forceinline__ float warp_row_sums(float (&v)[16], int l, int &row_out) {
-    float a8[8];
-    const bool h16 = l & 16;
-#pragma unroll
-    for (int t = 0; t < 8; t++) {
-        const float keep = h16 ? v[8 + t] : v[t], send = h16 ? v[t] : v[8 + t];
-        a8[t] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
-    }
-    float a4[4];
-    const bool h8 = l & 8;
-#pragma unroll
-    for (int t = 0; t < 4; t++) {
-        const float keep = h8 ? a8[4 + t] : a8[t], send = h8 ? a8[t] : a8[4 + t];
-        a4[t] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
-    }
-    float a2[2];
-    const bool h4 = l & 4;
-#pragma unroll
-    for (int t = 0; t < 2; t++) {
-        const float keep = h4 ? a4[2 + t] : a4[t], send = h4 ? a4[t] : a4[2 + t];
-        a2[t] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
-    }
-    const bool h2 = l & 2;
-    float a1 = (h2 ? a2[1] : a2[0]) + __shfl_xor_sync(0xffffffffu, h2 ? a2[0] : a2[1], 2);
-    a1 += __shfl_xor_sync(0xffffffffu, a1, 1);
-    row_out = 8 * ((l >> 4) & 1) + 4 * ((l >> 3) & 1) + 2 * ((l >> 2) & 1) + ((l >> 1) & 1);
-    return a1;
-}
-
 // Cross-warp column reduction of NR values per thread column (4 columns per
 // thread, 8 warps) into partial region `reg0` and the following ones.
 template <int NR>
@@ -268,17 +234,12 @@ __device__ __forceinline__ void cols_to_red(const T &t, float *red, int reg0, co
 #pragma unroll
         for (int c = 0; c < 4; c++) red[((reg0 + k) * 8 + t.w) * 128 + t.col(c)] = v[k][c];
 }
-__device__ __forceinline__ float pair_sum(uint64_t v) { return f2lo(v) + f2hi(v); }
 
 // Per-row sums over the thread's 4 columns of |value|, for the row pair's
 // low (even) and high (odd) rows.
 __device__ __forceinline__ void abs_row_sums(const uint64_t (&x)[4], float &lo, float &hi) {
     lo = (fabsf(f2lo(x[0])) + fabsf(f2lo(x[1]))) + (fabsf(f2lo(x[2])) + fabsf(f2lo(x[3])));
     hi = (fabsf(f2hi(x[0])) + fabsf(f2hi(x[1]))) + (fabsf(f2hi(x[2])) + fabsf(f2hi(x[3])));
-}
-
-__device__ __forceinline__ uint64_t clamp2(uint64_t v, float lim) {
-    return f2(fminf(fmaxf(f2lo(v), -lim), lim), fminf(fmaxf(f2hi(v), -lim), lim));
 }
 
 // Least-squares sums of the thread's columns: n_j += alpha_i z_ij X'_ij and
@@ -527,18 +488,10 @@ struct DecodeArgs {
     int fit_iters;
 };
 
-__device__ __forceinline__ bool slot_ok(const DecodeArgs &a, int slot) {
-    return slot >= 0 && slot < a.pool_slots;
-}
-
-// Producer: start the copies of the item (head h, batch entry b) into stage s
-// (one thread). An invalid slot completes the phase without data.
+// Producer: start the copies of the item (head h, batch entry b, a valid slot)
+// into stage s.
 __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s) {
     uint64_t *bar = &S.bars[s];
-    if (!slot_ok(a, slot)) {
-        mbar_arrive(bar);
-        return;
-    }
     Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
     const uint32_t nb = S.hbytes[h];
     const int hk = S.hkey[h];
@@ -647,30 +600,11 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     return true;
 }
 
-// (head, batch entry) of item = head * nb + entry, stepped by the grid stride
-// G = gq * nb + gr without divisions.
-struct Cursor {
-    int item, h, b;
-    __device__ __forceinline__ Cursor(int it, int nb) : item(it), h(it / nb), b(it - (it / nb) * nb) {}
-    __device__ __forceinline__ void step(int G, int gq, int gr, int nb) {
-        item += G;
-        h += gq;
-        b += gr;
-        if (b >= nb) {
-            b -= nb;
-            h++;
-        }
-    }
-};
-
 __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     const T t;
     const Smem S(smem);
-    const int G = gridDim.x, S_n = a.n_stages;
-    const int gq = G / a.nb, gr = G - gq * a.nb;
-    const int first = blockIdx.x;
-    if (first >= a.items) return;
+    if ((int)blockIdx.x >= a.items) return;
     const int grp = a.Hv / a.Hk;
     for (int h = t.tid; h < a.Hv; h += kThreads) {
         S.hoff[h] = a.tab.head_off[h];
@@ -678,105 +612,31 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
         S.hbits[h] = a.tab.head_bits[h];
         S.hkey[h] = (uint8_t)(h / grp);
     }
-    if (t.tid == kProducer) {
-        for (int s = 0; s < S_n; s++) mbar_init(&S.bars[s], 1);
+    if (t.tid == pipe::kProducer) {
+        for (int s = 0; s < a.n_stages; s++) mbar_init(&S.bars[s], 1);
         mbar_init_fence();
     }
     __syncthreads();
-    // With three or more stages a stage is refilled two items after its own item
-    // (its store has long finished reading it); with two stages, one item after.
-    const int lag = S_n >= 3 ? 2 : 1;
-    if (t.tid == kProducer) {
-        Cursor c0(first, a.nb);
-        for (int s = 0; s < S_n && c0.item < a.items; s++) {
-            issue(a, S, c0.h, c0.b, a.slots[c0.b], s);
-            c0.step(G, gq, gr, a.nb);
-        }
-    }
-    // iteration n >= lag refills stage (n - lag) mod S with item n - lag + S
-    Cursor cur(first, a.nb), iss(first + S_n * G, a.nb);
-    // scalars of the current item; the next item's are fetched one iteration ahead
-    int slot = a.slots[cur.b];
-    float alpha = a.gate[(size_t)cur.b * a.Hv + cur.h], beta = a.beta[(size_t)cur.b * a.Hv + cur.h];
-    int s = 0, is = 0;                    // stage of the current item, stage refilled next
-    uint32_t parity = 0;
-    for (int n = 0; cur.item < a.items; n++) {
-        // prefetch: next item's scalars (all threads), and the slot of the item
-        // this iteration will issue (producer)
-        Cursor nxt = cur;
-        nxt.step(G, gq, gr, a.nb);
-        int nslot = -1;
-        float nalpha = 0.f, nbeta = 0.f;
-        if (nxt.item < a.items) {
-            nslot = a.slots[nxt.b];
-            nalpha = a.gate[(size_t)nxt.b * a.Hv + nxt.h];
-            nbeta = a.beta[(size_t)nxt.b * a.Hv + nxt.h];
-        }
-        const bool do_issue = n >= lag && iss.item < a.items;
-        int islot = -1;
-        if (t.tid == kProducer && do_issue) islot = a.slots[iss.b];
-
-        const bool ok = mbar_wait(&S.bars[s], parity, kWaitCycles);
-        const bool valid = slot_ok(a, slot);
-        if (!valid && t.tid == 0) raise_error(a.err, STEPQ_ERR_SLOT_RANGE);
-        const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
-        // Refill the stage of an earlier item (its store was committed `lag`
-        // items ago) with the item S-1 ahead of it: S-1 items stay in flight.
-        const auto refill = [&]() {
-            if (t.tid == kProducer && do_issue) {
-                if (lag == 2) bulk_wait_read_all_but_one();
-                else bulk_wait_read_all();
-                issue(a, S, iss.h, iss.b, islot, is);
-            }
-        };
-        bool alive = true;
-        const int h = cur.h;
-        if (valid) {
-            float *y_out = a.y + ((size_t)cur.b * a.Hv + h) * 128;
+    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err};
+    pipe::run(
+        p, S.bars,
+        [&](int h, int b, int slot, int s) { issue(a, S, h, b, slot, s); },
+        [&](int h, int b, int, int s, bool ok, const auto &refill) {
+            const float2 gb = make_float2(a.gate[(size_t)b * a.Hv + h], a.beta[(size_t)b * a.Hv + h]);
+            const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
+            float *y_out = a.y + ((size_t)b * a.Hv + h) * 128;
             switch (S.hbits[h]) {
-            case 2: alive = decode_item<2>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
-            case 4: alive = decode_item<4>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
-            case 6: alive = decode_item<6>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
-            case 8: alive = decode_item<8>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
-            default: alive = decode_item<kPivot>(t, S, st, alpha, beta, y_out, a.fit_iters, ok, refill); break;
+            case 2: return decode_item<2>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
+            case 4: return decode_item<4>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
+            case 6: return decode_item<6>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
+            case 8: return decode_item<8>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
+            default: return decode_item<kPivot>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
             }
-        } else {
-            alive = !__syncthreads_or(!ok);
-            if (alive) refill();
-        }
-        if (!alive) {
-            if (t.tid == kProducer) {
-                raise_error(a.err, STEPQ_ERR_TIMEOUT);
-                // drain this CTA's copies still in flight (items n .. issued), with a bound
-                const int last = n < lag ? S_n - 1 : n - 1 - lag + S_n;
-                for (int m = n; m <= last; m++) {
-                    if (first + m * G >= a.items) break;
-                    mbar_wait(&S.bars[m % S_n], (uint32_t)(m / S_n) & 1u, kWaitCycles);
-                }
-                bulk_wait_all();
-            }
-            return;
-        }
-        __syncthreads();                                 // the page in stage s is final
-        if (t.tid == kProducer) {
-            if (valid) {
-                fence_async_smem();
-                bulk_store(a.pool + (uint64_t)slot * a.stride + S.hoff[h], st.page, S.hbytes[h]);
-            }
-            bulk_commit();
-        }
-        cur = nxt;
-        slot = nslot; alpha = nalpha; beta = nbeta;
-        if (n >= lag) {
-            iss.step(G, gq, gr, a.nb);
-            if (++is == S_n) is = 0;
-        }
-        if (++s == S_n) {
-            s = 0;
-            parity ^= 1u;
-        }
-    }
-    if (t.tid == kProducer) bulk_wait_all();
+        },
+        [&](int h, int slot, int s) {
+            bulk_store(a.pool + (uint64_t)slot * a.stride + S.hoff[h],
+                       S.stages + (size_t)s * a.stage_bytes, S.hbytes[h]);
+        });
 }
 
 // ---------------------------------------------------------- pack / unpack

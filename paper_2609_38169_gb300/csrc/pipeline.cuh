@@ -1,0 +1,153 @@
+// The persistent page pipeline shared by the fused decode kernels.
+//
+// Each CTA walks the items first, first + G, first + 2G, ... of one launch
+// (item = head * nb + batch entry, head-major so that concurrently resident
+// CTAs mostly work on one head). One producer thread keeps up to S-1 items in
+// flight: their copies land in a ring of S shared-memory stages and complete on
+// one mbarrier per stage. Every thread consumes the current stage, the page is
+// rewritten in place, and the producer writes it back with a bulk store.
+//
+// Every wait is bounded: a stage whose copies do not land within kWaitCycles
+// raises STEPQ_ERR_TIMEOUT (the CTA agrees on it at its first barrier of the
+// item), and the producer then waits, again with a bound, for this CTA's
+// copies still in flight before the CTA returns.
+#pragma once
+
+#include <cstdint>
+
+#include "async.cuh"
+#include "device.cuh"
+
+namespace stepq {
+namespace pipe {
+
+constexpr long long kWaitCycles = 2000000000LL;      // ~1 s at 2 GHz
+constexpr int kProducer = kThreads - 32;              // lane 0 of the last warp issues copies
+
+// (head, batch entry) of item = head * nb + entry, stepped by the grid stride
+// G = gq * nb + gr without divisions.
+struct Cursor {
+    int item, h, b;
+    __device__ __forceinline__ Cursor(int it, int nb) : item(it), h(it / nb), b(it - (it / nb) * nb) {}
+    __device__ __forceinline__ void step(int G, int gq, int gr, int nb) {
+        item += G;
+        h += gq;
+        b += gr;
+        if (b >= nb) {
+            b -= nb;
+            h++;
+        }
+    }
+};
+
+struct Shape {
+    int items, nb, n_stages;
+    const int32_t *slots;
+    int pool_slots;
+    unsigned int *err;
+};
+
+// Runs the item loop of this CTA (all threads call it; bars[0..S) initialised).
+//   issue(h, b, slot, s)      producer only: arrive with expect_tx on bars[s]
+//                             and start the item's copies into stage s
+//   process(h, b, slot, s, ok, refill) -> bool
+//                             all threads: the step on stage s; must call
+//                             refill() once, and return false from its first
+//                             CTA barrier (which takes the OR of !ok) if a copy
+//                             stalled
+//   store(h, slot, s)         producer only: write the final page back
+// An item whose slot id is out of range raises STEPQ_ERR_SLOT_RANGE; its stage
+// completes without data and nothing is written.
+template <class Issue, class Process, class Store>
+__device__ __forceinline__ void run(const Shape &p, uint64_t *bars, Issue &&issue, Process &&process,
+                                    Store &&store) {
+    const int tid = threadIdx.x;
+    const int G = gridDim.x, S_n = p.n_stages;
+    const int gq = G / p.nb, gr = G - gq * p.nb;
+    const int first = blockIdx.x;
+    const auto slot_ok = [&](int slot) { return slot >= 0 && slot < p.pool_slots; };
+    const auto start = [&](int h, int b, int slot, int s) {
+        if (slot_ok(slot)) issue(h, b, slot, s);
+        else mbar_arrive(&bars[s]);
+    };
+    // With three or more stages a stage is refilled two items after its own item
+    // (its store has long finished reading it); with two stages, one item after.
+    const int lag = S_n >= 3 ? 2 : 1;
+    if (tid == kProducer) {
+        Cursor c0(first, p.nb);
+        for (int s = 0; s < S_n && c0.item < p.items; s++) {
+            start(c0.h, c0.b, p.slots[c0.b], s);
+            c0.step(G, gq, gr, p.nb);
+        }
+    }
+    // iteration n >= lag refills stage (n - lag) mod S with item n - lag + S
+    Cursor cur(first, p.nb), iss(first + S_n * G, p.nb);
+    int slot = p.slots[cur.b];
+    int s = 0, is = 0;                    // stage of the current item, stage refilled next
+    uint32_t parity = 0;
+    for (int n = 0; cur.item < p.items; n++) {
+        // prefetch: the next item's slot (all threads) and the slot of the item
+        // this iteration will issue (producer)
+        Cursor nxt = cur;
+        nxt.step(G, gq, gr, p.nb);
+        const int nslot = nxt.item < p.items ? p.slots[nxt.b] : -1;
+        const bool do_issue = n >= lag && iss.item < p.items;
+        int islot = -1;
+        if (tid == kProducer && do_issue) islot = p.slots[iss.b];
+
+        const bool ok = mbar_wait(&bars[s], parity, kWaitCycles);
+        const bool valid = slot_ok(slot);
+        if (!valid && tid == 0) raise_error(p.err, STEPQ_ERR_SLOT_RANGE);
+        // Refill the stage of an earlier item (its store was committed `lag`
+        // items ago) with the item S-1 ahead of it: S-1 items stay in flight.
+        const auto refill = [&start, tid, do_issue, lag, islot, iss, is]() {
+            if (tid == kProducer && do_issue) {
+                if (lag == 2) bulk_wait_read_all_but_one();
+                else bulk_wait_read_all();
+                start(iss.h, iss.b, islot, is);
+            }
+        };
+        bool alive;
+        if (valid) {
+            alive = process(cur.h, cur.b, slot, s, ok, refill);
+        } else {
+            alive = !__syncthreads_or(!ok);
+            if (alive) refill();
+        }
+        if (!alive) {
+            if (tid == kProducer) {
+                raise_error(p.err, STEPQ_ERR_TIMEOUT);
+                // drain this CTA's copies still in flight (items n .. issued), with a bound
+                const int last = n < lag ? S_n - 1 : n - 1 - lag + S_n;
+                for (int m = n; m <= last; m++) {
+                    if (first + m * G >= p.items) break;
+                    mbar_wait(&bars[m % S_n], (uint32_t)(m / S_n) & 1u, kWaitCycles);
+                }
+                bulk_wait_all();
+            }
+            return;
+        }
+        __syncthreads();                                 // the page in stage s is final
+        if (tid == kProducer) {
+            if (valid) {
+                fence_async_smem();
+                store(cur.h, slot, s);
+            }
+            bulk_commit();
+        }
+        cur = nxt;
+        slot = nslot;
+        if (n >= lag) {
+            iss.step(G, gq, gr, p.nb);
+            if (++is == S_n) is = 0;
+        }
+        if (++s == S_n) {
+            s = 0;
+            parity ^= 1u;
+        }
+    }
+    if (tid == kProducer) bulk_wait_all();
+}
+
+}  // namespace pipe
+}  // namespace stepq

@@ -1,12 +1,10 @@
-// Row-unit (KDA) decode step, pool pack/unpack and the calibration distortion
-// kernel (sm_103a). Head units (GDN) run the pipelined kernels of heads.cu.
+// Row-unit (KDA) pool pack/unpack and the calibration distortion kernel
+// (sm_103a), and the dispatch of the decode step: head units (GDN) run the
+// pipelined kernel of heads.cu, row units the one of rows.cu.
 //
-// One 256-thread CTA owns one (slot, value head) page: it stages the packed
-// head segment in shared memory with 128-bit loads, reconstructs the tile into
-// registers, applies the gated Delta update, emits the readout, refits the
-// dual-axis scales and writes the repacked segment back in place (App. C.3
-// steps 1-7; the fusion of Sec. 4.4). Nothing of the tile leaves the SM
-// between the read and the write of its page.
+// One 256-thread CTA owns one (slot, value head) page: it stages the head
+// segment in shared memory with 128-bit loads, holds the tile in registers,
+// fits the dual-axis scales and writes the packed segment (App. C.3 steps 4-6).
 //
 // Numerical contract (shared with the CPU oracle, which restates it in fp64):
 // the tile X is fp32; r_i = fp16(clamp(sqrt(m_i) * w_i^(-1/2), 2^-14, 65504));
@@ -199,109 +197,6 @@ __device__ __forceinline__ void load_row_meta(const Lane &L, const TileSmem &S,
 
 __device__ __forceinline__ void copy16(uint4 *dst, const uint4 *src, int n16, int tid) {
     for (int e = tid; e < n16; e += kThreads) dst[e] = src[e];
-}
-
-// ------------------------------------------------------------------ decode
-struct DecodeArgs {
-    uint8_t *pool;
-    uint64_t stride;
-    int pool_slots;
-    const int32_t *slots;
-    LayerTables tab;
-    Shape sh;
-    const float *q, *k, *v, *beta, *gate;
-    float *y;
-    unsigned int *err;
-};
-
-__global__ void __launch_bounds__(kThreads, 2) decode_step_kernel(DecodeArgs a) {
-    extern __shared__ __align__(16) uint8_t smem[];
-    const Lane L;
-    const TileSmem S(smem);
-    const int Hv = a.sh.Hv, Hk = a.sh.Hk;
-    const int b = blockIdx.x / Hv, h = blockIdx.x - b * Hv;
-    const int slot = a.slots[b];
-    if (slot < 0 || slot >= a.pool_slots) {
-        if (L.tid == 0) raise_error(a.err, STEPQ_ERR_SLOT_RANGE);
-        return;
-    }
-    uint8_t *gpage = a.pool + (uint64_t)slot * a.stride + a.tab.head_off[h];
-    const int nbytes = (int)a.tab.head_bytes[h];
-    const int has_scales = a.tab.head_bits[h] != kPivot;
-    copy16((uint4 *)S.page, (const uint4 *)gpage, nbytes >> 4, L.tid);
-    load_row_meta(L, S, a.tab, h);
-    if (L.tid < 128) {
-        const int hk = h / (Hv / Hk);
-        S.qv[L.tid] = a.q[((size_t)b * Hk + hk) * 128 + L.tid];
-        S.kv[L.tid] = a.k[((size_t)b * Hk + hk) * 128 + L.tid];
-        S.gv[L.tid] = a.sh.gate_per_row ? a.gate[((size_t)b * Hv + h) * 128 + L.tid]
-                                        : a.gate[(size_t)b * Hv + h];
-    }
-    const float beta = a.beta[(size_t)b * Hv + h];
-    __syncthreads();
-
-    // Steps 1-2a: reconstruct P = D S_hat (S_hat_ij = r_i c_j z_ij, or FP16) and
-    // retrieve u = k^T P.
-    float x[4][16];
-    float cj[16];
-    const uint16_t *page_r = (const uint16_t *)S.page;
-    const uint16_t *page_c = (const uint16_t *)(S.page + 256);
-#pragma unroll
-    for (int j = 0; j < 16; j++) cj[j] = has_scales ? f16_val(page_c[L.col0() + j]) : 1.f;
-    float acc[1][16];
-#pragma unroll
-    for (int j = 0; j < 16; j++) acc[0][j] = 0.f;
-#pragma unroll
-    for (int t = 0; t < 4; t++) {
-        const int i = L.row(t);
-        const int bits = S.rbits[i];
-        float vals[16];
-        load_row16(S.page + S.roff[i], bits, L.cg, vals);
-        const float d = S.gv[i], ki = S.kv[i];
-        if (bits == kPivot) {
-#pragma unroll
-            for (int j = 0; j < 16; j++) x[t][j] = d * vals[j];
-        } else {
-            const float zs = a.sh.unit_kind ? (float)(1 << (8 - bits)) : 1.f;
-            const float s = d * (f16_val(page_r[i]) * zs);
-#pragma unroll
-            for (int j = 0; j < 16; j++) x[t][j] = s * (cj[j] * vals[j]);
-        }
-#pragma unroll
-        for (int j = 0; j < 16; j++) acc[0][j] += ki * x[t][j];
-    }
-    float *colU = S.col + 512;    // [4][128] of S.col belong to fit_and_pack
-    column_reduce<1, false>(L, acc, S.red, colU);
-
-    // Step 2b-3: X = P + beta k (v - u)^T; y = X^T q (before requantization).
-    float delta[16];
-#pragma unroll
-    for (int j = 0; j < 16; j++) {
-        const int c = L.col0() + j;
-        delta[j] = a.v[((size_t)b * Hv + h) * 128 + c] - colU[c];
-        acc[0][j] = 0.f;
-    }
-    float msum[4];
-#pragma unroll
-    for (int t = 0; t < 4; t++) {
-        const int i = L.row(t);
-        const float bk = beta * S.kv[i], qi = S.qv[i];
-        float s = 0.f;
-#pragma unroll
-        for (int j = 0; j < 16; j++) {
-            const float X = fmaf(bk, delta[j], x[t][j]);
-            x[t][j] = X;
-            acc[0][j] += qi * X;
-            s += fabsf(X);
-        }
-        msum[t] = row_allreduce(s);
-    }
-    column_reduce<1, false>(L, acc, S.red, colU);
-    if (L.tid < 128) a.y[((size_t)b * Hv + h) * 128 + L.tid] = colU[L.tid];
-
-    // Steps 4-6: refit and pack; step 7: write the page back in place.
-    fit_and_pack(L, S, x, msum, a.sh.unit_kind, has_scales, a.sh.fit_iters);
-    copy16((uint4 *)gpage, (const uint4 *)S.page, nbytes >> 4, L.tid);
 }
 
 // ---------------------------------------------------------- quantize / dequantize
@@ -500,9 +395,7 @@ static stepq_status prepare(int dev) {
     if (dev < 0) cudaGetDevice(&dev);
     if (dev < 0 || dev >= 64) return STEPQ_ERR_CUDA;
     if (!g_attr_set[dev]) {
-        if (cudaFuncSetAttribute(decode_step_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kSmemBytes) != cudaSuccess ||
-            cudaFuncSetAttribute(quantize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(quantize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kSmemBytes) != cudaSuccess ||
             cudaFuncSetAttribute(dequantize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kSmemBytes) != cudaSuccess ||
@@ -524,12 +417,7 @@ stepq_status launch_decode(const stepq_plan *p, int layer, uint8_t *pool, int po
                            cudaStream_t s) {
     if (p->cfg.gate_kind == STEPQ_GATE_SCALAR)
         return launch_decode_heads(p, layer, pool, pool_slots, slots, B, q, k, v, beta, gate, y, s);
-    stepq_status st = prepare(p->device);
-    if (st != STEPQ_OK) return st;
-    DecodeArgs a{pool, p->slot_stride, pool_slots, slots, p->layer(layer), p->shape(),
-                 q, k, v, beta, gate, y, device_error_word()};
-    decode_step_kernel<<<(unsigned)B * p->cfg.n_value_heads, kThreads, kSmemBytes, s>>>(a);
-    return launched();
+    return launch_decode_rows(p, layer, pool, pool_slots, slots, B, q, k, v, beta, gate, y, s);
 }
 
 stepq_status launch_quantize(const stepq_plan *p, int layer, const float *states,
