@@ -1,8 +1,8 @@
 // Comparison decode kernels written in the same build: the FP32-state step
 // (the serving default the paper measures against, Sec. 5.1) and the uniform
 // rowwise-absmax INT-b state (App. B.5: per key row an FP16 scale absmax/q_b in
-// [2^-14, 65504], nearest codes in [-q_b, q_b]). Same tile mapping and
-// reductions as the STEPQuant kernel, one CTA per (slot, value head).
+// [2^-14, 65504], nearest codes in [-q_b, q_b]) pack/unpack. One CTA per
+// (slot, value head); the pipelined INT-b decode step is in intb.cu.
 #include "device.cuh"
 #include "internal.h"
 
@@ -25,7 +25,6 @@ struct BaseArgs {
     unsigned int *err;
 };
 
-constexpr int kBaseSmem = 2 * 8 * 128 * 4 + 4 * 128 * 4 + 3 * 128 * 4 + 16896;
 
 // Shared part of both baselines after the state P = D S is in registers:
 // u = k^T P, X = P + beta k (v - u)^T, y = X^T q.
@@ -161,35 +160,6 @@ __device__ __forceinline__ void intb_unpack(const Lane &L, const uint8_t *page, 
     }
 }
 
-__global__ void __launch_bounds__(kThreads, 2) intb_decode_kernel(BaseArgs a) {
-    extern __shared__ __align__(16) uint8_t smem[];
-    float *red = (float *)smem, *col = red + 2048, *qv = col + 512, *kv = qv + 128, *gv = kv + 128;
-    uint8_t *page = (uint8_t *)(gv + 128);
-    const Lane L;
-    int b, h;
-    const int slot = unit_slot(a, b, h);
-    if (slot < 0) return;
-    uint8_t *gpage = a.pool + (uint64_t)slot * a.slot_bytes + a.layer_off + h * a.head_bytes;
-    for (int e = L.tid; e < (int)(a.head_bytes >> 4); e += kThreads)
-        ((uint4 *)page)[e] = ((const uint4 *)gpage)[e];
-    load_vectors(L, a, b, h, qv, kv, gv);
-    __syncthreads();
-    float x[4][16];
-    intb_unpack(L, page, a.bits, x);
-#pragma unroll
-    for (int t = 0; t < 4; t++) {
-        const float d = gv[L.row(t)];
-#pragma unroll
-        for (int j = 0; j < 16; j++) x[t][j] *= d;
-    }
-    delta_update_readout(L, x, red, col, qv, kv, a.v + ((size_t)b * a.Hv + h) * 128,
-                         a.beta[(size_t)b * a.Hv + h], a.y + ((size_t)b * a.Hv + h) * 128);
-    intb_pack(L, x, page, a.bits);     // old page fully consumed before the reductions
-    __syncthreads();
-    for (int e = L.tid; e < (int)(a.head_bytes >> 4); e += kThreads)
-        ((uint4 *)gpage)[e] = ((const uint4 *)page)[e];
-}
-
 __global__ void __launch_bounds__(kThreads, 2) intb_quantize_kernel(BaseArgs a) {
     extern __shared__ __align__(16) uint8_t smem[];
     uint8_t *page = smem;
@@ -237,19 +207,6 @@ __global__ void __launch_bounds__(kThreads, 2) intb_dequantize_kernel(BaseArgs a
 }
 
 // ------------------------------------------------------------------ launchers
-static stepq_status set_smem_once() {
-    static bool done[64];
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return STEPQ_ERR_CUDA;
-    if (!done[dev]) {
-        if (cudaFuncSetAttribute(intb_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kBaseSmem) != cudaSuccess)
-            return STEPQ_ERR_CUDA;
-        done[dev] = true;
-    }
-    return STEPQ_OK;
-}
-
 static BaseArgs base_args(const stepq_config *cfg, int bits, int layer, uint8_t *pool,
                           int pool_slots, const int32_t *slots) {
     BaseArgs a{};
@@ -277,18 +234,6 @@ stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool,
     BaseArgs a = base_args(cfg, 32, layer, (uint8_t *)pool, pool_slots, slots);
     a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
     fp32_decode_kernel<<<(unsigned)B * cfg->n_value_heads, kThreads, 2 * 8 * 128 * 4 + 7 * 128 * 4, s>>>(a);
-    return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;
-}
-
-stepq_status launch_intb_decode(const stepq_config *cfg, int bits, int layer, uint8_t *pool,
-                                int pool_slots, const int32_t *slots, int B, const float *q,
-                                const float *k, const float *v, const float *beta,
-                                const float *gate, float *y, cudaStream_t s) {
-    stepq_status st = set_smem_once();
-    if (st != STEPQ_OK) return st;
-    BaseArgs a = base_args(cfg, bits, layer, pool, pool_slots, slots);
-    a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
-    intb_decode_kernel<<<(unsigned)B * cfg->n_value_heads, kThreads, kBaseSmem, s>>>(a);
     return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;
 }
 
