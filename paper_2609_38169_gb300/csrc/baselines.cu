@@ -1,8 +1,7 @@
-// Comparison decode kernels written in the same build: the FP32-state step
-// (the serving default the paper measures against, Sec. 5.1) and the uniform
-// rowwise-absmax INT-b state (App. B.5: per key row an FP16 scale absmax/q_b in
-// [2^-14, 65504], nearest codes in [-q_b, q_b]) pack/unpack. One CTA per
-// (slot, value head); the pipelined INT-b decode step is in intb.cu.
+// Pack/unpack of the uniform rowwise-absmax INT-b comparison state (App. B.5:
+// per key row an FP16 scale absmax/q_b in [2^-14, 65504], nearest codes in
+// [-q_b, q_b]). One CTA per (slot, value head); the pipelined INT-b decode step
+// is in intb.cu and the FP32-state step in fp32.cu.
 #include "device.cuh"
 #include "internal.h"
 
@@ -11,7 +10,7 @@ namespace stepq {
 size_t intb_head_bytes(int bits) { return 256 + (size_t)kD * 16 * bits; }
 
 struct BaseArgs {
-    uint8_t *pool;              // fp32 pool (as bytes) or INT-b pool
+    uint8_t *pool;              // INT-b pool
     uint64_t slot_bytes;        // bytes per slot page
     uint64_t layer_off;         // byte offset of the layer inside a page
     uint64_t head_bytes;        // bytes per head segment
@@ -25,43 +24,6 @@ struct BaseArgs {
     unsigned int *err;
 };
 
-
-// Shared part of both baselines after the state P = D S is in registers:
-// u = k^T P, X = P + beta k (v - u)^T, y = X^T q.
-__device__ __forceinline__ void delta_update_readout(const Lane &L, float (&x)[4][16], float *red,
-                                                     float *col, const float *qv, const float *kv,
-                                                     const float *vg, float beta, float *yg) {
-    float acc[1][16];
-#pragma unroll
-    for (int j = 0; j < 16; j++) acc[0][j] = 0.f;
-#pragma unroll
-    for (int t = 0; t < 4; t++) {
-        const float ki = kv[L.row(t)];
-#pragma unroll
-        for (int j = 0; j < 16; j++) acc[0][j] += ki * x[t][j];
-    }
-    column_reduce<1, false>(L, acc, red, col);
-    float delta[16];
-#pragma unroll
-    for (int j = 0; j < 16; j++) {
-        delta[j] = vg[L.col0() + j] - col[L.col0() + j];
-        acc[0][j] = 0.f;
-    }
-#pragma unroll
-    for (int t = 0; t < 4; t++) {
-        const int i = L.row(t);
-        const float bk = beta * kv[i], qi = qv[i];
-#pragma unroll
-        for (int j = 0; j < 16; j++) {
-            const float X = fmaf(bk, delta[j], x[t][j]);
-            x[t][j] = X;
-            acc[0][j] += qi * X;
-        }
-    }
-    column_reduce<1, false>(L, acc, red, col + 128);
-    if (L.tid < 128) yg[L.tid] = col[128 + L.tid];
-}
-
 __device__ __forceinline__ int unit_slot(const BaseArgs &a, int &b, int &h) {
     b = blockIdx.x / a.Hv;
     h = blockIdx.x - b * a.Hv;
@@ -71,53 +33,6 @@ __device__ __forceinline__ int unit_slot(const BaseArgs &a, int &b, int &h) {
         return -1;
     }
     return slot;
-}
-
-__device__ __forceinline__ void load_vectors(const Lane &L, const BaseArgs &a, int b, int h,
-                                             float *qv, float *kv, float *gv) {
-    if (L.tid < 128) {
-        const int hk = h / (a.Hv / a.Hk);
-        qv[L.tid] = a.q[((size_t)b * a.Hk + hk) * 128 + L.tid];
-        kv[L.tid] = a.k[((size_t)b * a.Hk + hk) * 128 + L.tid];
-        gv[L.tid] = a.gate_per_row ? a.gate[((size_t)b * a.Hv + h) * 128 + L.tid]
-                                   : a.gate[(size_t)b * a.Hv + h];
-    }
-}
-
-// ---------------------------------------------------------------- FP32 state
-__global__ void __launch_bounds__(kThreads, 2) fp32_decode_kernel(BaseArgs a) {
-    extern __shared__ __align__(16) uint8_t smem[];
-    float *red = (float *)smem, *col = red + 2048, *qv = col + 512, *kv = qv + 128, *gv = kv + 128;
-    const Lane L;
-    int b, h;
-    const int slot = unit_slot(a, b, h);
-    if (slot < 0) return;
-    float *S = (float *)(a.pool + (uint64_t)slot * a.slot_bytes + a.layer_off + h * a.head_bytes);
-    load_vectors(L, a, b, h, qv, kv, gv);
-    __syncthreads();
-    float x[4][16];
-#pragma unroll
-    for (int t = 0; t < 4; t++) {
-        const float d = gv[L.row(t)];
-        const float4 *src = (const float4 *)(S + L.row(t) * 128 + L.col0());
-#pragma unroll
-        for (int e = 0; e < 4; e++) {
-            const float4 f = src[e];
-            x[t][4 * e] = d * f.x;
-            x[t][4 * e + 1] = d * f.y;
-            x[t][4 * e + 2] = d * f.z;
-            x[t][4 * e + 3] = d * f.w;
-        }
-    }
-    delta_update_readout(L, x, red, col, qv, kv, a.v + ((size_t)b * a.Hv + h) * 128,
-                         a.beta[(size_t)b * a.Hv + h], a.y + ((size_t)b * a.Hv + h) * 128);
-#pragma unroll
-    for (int t = 0; t < 4; t++) {
-        float4 *dst = (float4 *)(S + L.row(t) * 128 + L.col0());
-#pragma unroll
-        for (int e = 0; e < 4; e++)
-            dst[e] = make_float4(x[t][4 * e], x[t][4 * e + 1], x[t][4 * e + 2], x[t][4 * e + 3]);
-    }
 }
 
 // ---------------------------------------------------------------- INT-b state
@@ -210,11 +125,11 @@ __global__ void __launch_bounds__(kThreads, 2) intb_dequantize_kernel(BaseArgs a
 static BaseArgs base_args(const stepq_config *cfg, int bits, int layer, uint8_t *pool,
                           int pool_slots, const int32_t *slots) {
     BaseArgs a{};
-    const uint64_t hb = bits == 32 ? (uint64_t)kN * 4 : intb_head_bytes(bits);
+    const uint64_t hb = intb_head_bytes(bits);
     const uint64_t per_layer = hb * (uint64_t)cfg->n_value_heads;
     const uint64_t page = per_layer * (uint64_t)cfg->n_layers;
     a.pool = pool;
-    a.slot_bytes = bits == 32 ? page : (page + 255) / 256 * 256;
+    a.slot_bytes = (page + 255) / 256 * 256;
     a.layer_off = per_layer * (uint64_t)layer;
     a.head_bytes = hb;
     a.pool_slots = pool_slots;
@@ -225,16 +140,6 @@ static BaseArgs base_args(const stepq_config *cfg, int bits, int layer, uint8_t 
     a.bits = bits;
     a.err = device_error_word();
     return a;
-}
-
-stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool, int pool_slots,
-                                const int32_t *slots, int B, const float *q, const float *k,
-                                const float *v, const float *beta, const float *gate, float *y,
-                                cudaStream_t s) {
-    BaseArgs a = base_args(cfg, 32, layer, (uint8_t *)pool, pool_slots, slots);
-    a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
-    fp32_decode_kernel<<<(unsigned)B * cfg->n_value_heads, kThreads, 2 * 8 * 128 * 4 + 7 * 128 * 4, s>>>(a);
-    return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;
 }
 
 stepq_status launch_intb_quantize(const stepq_config *cfg, int bits, int layer,
