@@ -132,9 +132,13 @@ void stepq_plan_destroy(stepq_plan *plan);
 /* ----------------------------------------------------------------- device path
  * Pool: device, pool_slots * slot_stride bytes, 256-byte aligned. Slot page s
  * starts at pool + s * slot_stride and holds every (layer, head) segment:
- *   integer head unit: r[128] fp16 | c[128] fp16 | 128 rows x 16b bytes
- *   FP16 pivot head:   128 rows x 128 fp16
- *   row-unit head:     r[128] fp16 | c[128] fp16 | row i: 16*b_i bytes (b_i = 16: fp16 row)
+ *   integer head unit: r[128] fp16 | c[128] fp16 | codes in band-major chunks:
+ *                      for band w = 0..7 (rows 16w..16w+15) and column j, the
+ *                      band's 16 codes of column j in 2b bytes
+ *   FP16 pivot head:   the same chunk order of fp16 values (32 bytes per chunk)
+ *   row-unit head:     r[128] fp16 | c[128] fp16 | the rows, 16*b_i bytes each
+ *                      (b_i = 16: fp16 row), stored by decreasing width, rows of
+ *                      equal width in index order
  * Codes are offset binary u = q + 2^(b-1), packed LSB-first per row; row units
  * reconstruct with z = 2^(8-b_i) q (App. C.1).
  * layer: 0..L-1 for one layer, or -1 for every layer (quantize/dequantize only).

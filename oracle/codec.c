@@ -27,9 +27,10 @@
  *                      the 16 codes of rows 16w.. in that column (2b bytes)
  *   pivot head unit:   the same band-major order of fp16 values (32 bytes
  *                      per band column), no scales
- *   row-unit head:     r[128] fp16 | c[128] fp16 | row i: 16 b_i bytes with the
- *                      codes of columns 0..127 (b_i = 16 marks an FP16 pivot
- *                      row, 256 bytes)
+ *   row-unit head:     r[128] fp16 | c[128] fp16 | then the rows, each 16 b_i
+ *                      bytes with the codes of columns 0..127 (b_i = 16 marks
+ *                      an FP16 pivot row, 256 bytes), stored by decreasing
+ *                      width, rows of equal width in index order
  */
 #include <math.h>
 #include <stdlib.h>
@@ -74,9 +75,10 @@ static size_t elem_stream(int unit_kind, const int8_t *rb, int i, int j, int *bi
         *bitpos = (i % 16) * b;
         return base + chunk * 2 * (size_t)b;
     }
-    size_t off = 512;
-    for (int t = 0; t < i; t++)
-        off += 16 * (size_t)rb[t];
+    size_t off = 512;                      /* rows of larger width, then earlier rows of width b */
+    for (int t = 0; t < OR_D; t++)
+        if (rb[t] > b || (rb[t] == b && t < i))
+            off += 16 * (size_t)rb[t];
     *bitpos = j * b;
     return off;
 }

@@ -26,6 +26,7 @@ struct LayerTables {
     const uint8_t *head_bits; // [Hv] head width, 16 for a pivot head, 0 for row units
     const uint8_t *row_bits;  // [Hv][128]
     const uint32_t *row_off;  // [Hv][128] payload offset of row i within the head segment
+    const uint32_t *row_slot; // [Hv][128] s-th stored row: offset | width << 16 | row << 24
 };
 
 struct Shape {
@@ -57,12 +58,13 @@ struct stepq_plan {
     uint8_t *d_head_bits = nullptr;
     uint8_t *d_row_bits = nullptr;
     uint32_t *d_row_off = nullptr;
+    uint32_t *d_row_slot = nullptr;
 
     stepq::LayerTables layer(int l) const {
         const size_t Hv = (size_t)cfg.n_value_heads;
         return {d_w2 + l * Hv * stepq::kD, d_wis + l * Hv * stepq::kD, d_head_off + l * Hv,
                 d_head_bytes + l * Hv, d_head_bits + l * Hv, d_row_bits + l * Hv * stepq::kD,
-                d_row_off + l * Hv * stepq::kD};
+                d_row_off + l * Hv * stepq::kD, d_row_slot + l * Hv * stepq::kD};
     }
     stepq::Shape shape() const {
         return {cfg.n_key_heads, cfg.n_value_heads, cfg.n_layers,

@@ -283,7 +283,7 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
 
     // Packed layout: head segments in (layer, head) order, stride rounded to 256 B.
     std::vector<uint8_t> head_bits(heads), row_bits(heads * kD);
-    std::vector<uint32_t> row_off(heads * kD);
+    std::vector<uint32_t> row_off(heads * kD), row_slot(heads * kD, 0);
     p->head_off.resize(heads);
     p->head_bytes.resize(heads);
     uint64_t off = 0;
@@ -298,12 +298,21 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
             }
             bytes = b == kPivot ? 256u * kD : 512u + 16u * b * kD;
         } else {
+            // rows by decreasing width, equal widths in index order; slot s of
+            // the head is the s-th row stored: offset | width << 16 | row << 24
             head_bits[h] = 0;
-            bytes = 512;
+            int order[kD];
             for (int i = 0; i < kD; i++) {
-                int b = p->unit_bits[h * kD + i];
-                row_bits[h * kD + i] = (uint8_t)b;
+                order[i] = i;
+                row_bits[h * kD + i] = (uint8_t)p->unit_bits[h * kD + i];
+            }
+            std::stable_sort(order, order + kD,
+                             [&](int x, int y) { return row_bits[h * kD + x] > row_bits[h * kD + y]; });
+            bytes = 512;
+            for (int s = 0; s < kD; s++) {
+                const int i = order[s], b = row_bits[h * kD + i];
                 row_off[h * kD + i] = bytes;
+                row_slot[h * kD + s] = bytes | ((uint32_t)b << 16) | ((uint32_t)i << 24);
                 bytes += 16u * b;
             }
         }
@@ -325,7 +334,7 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
     size_t o_w2 = 0, o_wis = align(o_w2 + heads * kD * 4), o_off = align(o_wis + heads * kD * 4),
            o_hb = align(o_off + heads * 8), o_hbits = align(o_hb + heads * 4),
            o_rbits = align(o_hbits + heads), o_roff = align(o_rbits + heads * kD),
-           total = align(o_roff + heads * kD * 4);
+           o_rslot = align(o_roff + heads * kD * 4), total = align(o_rslot + heads * kD * 4);
     std::vector<uint8_t> host(total, 0);
     std::memcpy(host.data() + o_w2, w2.data(), heads * kD * 4);
     std::memcpy(host.data() + o_wis, wis.data(), heads * kD * 4);
@@ -334,6 +343,7 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
     std::memcpy(host.data() + o_hbits, head_bits.data(), heads);
     std::memcpy(host.data() + o_rbits, row_bits.data(), heads * kD);
     std::memcpy(host.data() + o_roff, row_off.data(), heads * kD * 4);
+    std::memcpy(host.data() + o_rslot, row_slot.data(), heads * kD * 4);
     int n_dev = 0;
     if (cudaGetDeviceCount(&n_dev) != cudaSuccess || n_dev == 0) {
         cudaGetLastError();          // host-only plan: its device calls return STEPQ_ERR_CUDA
@@ -355,6 +365,7 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
     p->d_head_bits = base + o_hbits;
     p->d_row_bits = base + o_rbits;
     p->d_row_off = (uint32_t *)(base + o_roff);
+    p->d_row_slot = (uint32_t *)(base + o_rslot);
     *out = p;
     return STEPQ_OK;
 }

@@ -1,19 +1,21 @@
 // Row-unit (KDA, per-key-channel gate) decode step: the persistent, bulk-async
 // pipelined kernel over row-major pages with one width per key row.
 //
-// Tile mapping: warp w owns key rows 16w..16w+15; lane l owns the value
-// columns 4l..4l+3. All lanes of a warp work on the same row at a time, so the
-// row's width is uniform across the warp (no divergence) and a lane's 4 codes
-// are one word (8-bit), half-word (4-bit), byte (2-bit), three bytes (6-bit,
-// assembled from two words) or four FP16 values (pivot row). A thread holds its
-// 16 rows x 2 column pairs as packed f32x2 registers: column constants of a lane
-// are adjacent in shared memory, per-row constants are stored as duplicated
-// pairs and read with broadcast loads.
+// Rows are stored by decreasing width, so the kernel works in storage order:
+// warp w owns the stored rows (slots) 16w..16w+15 and lane l the value columns
+// 4l..4l+3. All lanes of a warp read the same row at a time, so a row's width
+// is uniform across the warp and a lane's 4 codes are one contiguous 4b-bit
+// segment of the row. A thread holds 8 slot pairs x 4 columns as packed f32x2
+// registers: per-row constants of a pair are adjacent in shared memory (one
+// 128-bit load serves two pairs), column constants are duplicated pairs kept
+// in registers. Widths are handled with runtime shifts and masks (one funnel
+// shift per row segment), which keeps the unrolled code small; FP16 pivot rows
+// take an out-of-line path.
 //
 // Per row i the tile holds Z with X_ij = a_i Z_ij: a_i = d_i r_i zs_i and
 // Z = c_j q_ij for an integer row (zs_i = 2^(8 - b_i), the normalised codebook
 // of App. C.1), a_i = d_i and Z = the FP16 value for a pivot row. Pivot rows
-// stay out of the column fit (rho a = 1, mu = alpha = 0).
+// stay out of the column fit (rho a = 1, mu = alpha = qmax = 0).
 #include "async.cuh"
 #include "device.cuh"
 #include "internal.h"
@@ -23,7 +25,7 @@
 namespace stepq {
 namespace rk {
 
-constexpr int kVecBytes = 6 * 512 + 512 + 128;         // q k v gate w2 wis | row_off | row_bits
+constexpr int kVecBytes = 7 * 512;                     // q k v gate w2 wis | row slots
 
 // ------------------------------------------------------------ shared layout
 constexpr int kOffBars = 0;                            // uint64 [8]
@@ -33,9 +35,11 @@ constexpr int kOffColC = kOffRed + 3 * 8 * 128 * 4;    // float [128] c_j (start
 constexpr int kOffColM = kOffColC + 512;               // u32 [128] bits of max_i fp32(|X'_ij| mu_i)
 constexpr int kOffColD = kOffColM + 512;               // float [128] delta_j
 constexpr int kOffColG = kOffColD + 512;               // float [128] 1/c_j
-constexpr int kOffRows = kOffColG + 512;               // float4 [4][128] per-row constants
+constexpr int kNRowVec = 10;                           // per-row float vectors
+constexpr int kOffRows = kOffColG + 512;               // float [kNRowVec][128]
+constexpr int kOffInfo = kOffRows + kNRowVec * 512;    // uint2 [128]: (row slot, pack bias)
 constexpr int kMaxHv = 256;                            // value heads per layer (launch check)
-constexpr int kOffHead = kOffRows + 4 * 128 * 16;      // u64 off | u32 bytes | u8 key head
+constexpr int kOffHead = kOffInfo + 128 * 8;           // u64 off | u32 bytes | u8 key head
 constexpr int kOffStages = (kOffHead + kMaxHv * 13 + 127) / 128 * 128;
 
 struct Smem {
@@ -43,10 +47,10 @@ struct Smem {
     int *flags;
     float *red, *colC, *colD, *colG;
     uint32_t *colM;
-    float4 *rowK;   // (kappa, kappa, beta k / a, beta k / a), kappa = k a
-    float4 *rowQ;   // (q a, q a, a, a)
-    float4 *rowF;   // (rho a, rho a, alpha, alpha), alpha = w^2 (r zs)^2
-    float4 *rowM;   // (mu, mu, qmax, qmax): 1/qmax of the row's width (0 for pivots)
+    // per-row constants: kappa = k a, beta k / a, q a, a, rho a, alpha = w^2 (r zs)^2,
+    // mu = 1/qmax, qmax, the decode offset -(1.5*2^23 + 2^(b-1)) and 1.5*2^23 + 2^(b-1)
+    float *rKap, *rBkp, *rQa, *rA, *rRho, *rAl, *rMu, *rQm, *rOff, *rMb;
+    uint2 *rInfo;
     uint64_t *hoff;
     uint32_t *hbytes;
     uint8_t *hkey;
@@ -59,10 +63,10 @@ struct Smem {
         colM = (uint32_t *)(s + kOffColM);
         colD = (float *)(s + kOffColD);
         colG = (float *)(s + kOffColG);
-        rowK = (float4 *)(s + kOffRows);
-        rowQ = rowK + 128;
-        rowF = rowK + 256;
-        rowM = rowK + 384;
+        float *r = (float *)(s + kOffRows);
+        rKap = r; rBkp = r + 128; rQa = r + 256; rA = r + 384; rRho = r + 512;
+        rAl = r + 640; rMu = r + 768; rQm = r + 896; rOff = r + 1024; rMb = r + 1152;
+        rInfo = (uint2 *)(s + kOffInfo);
         hoff = (uint64_t *)(s + kOffHead);
         hbytes = (uint32_t *)(s + kOffHead + kMaxHv * 8);
         hkey = s + kOffHead + kMaxHv * 12;
@@ -73,8 +77,7 @@ struct Smem {
 struct Stage {
     uint8_t *page;
     float *q, *k, *v, *gate, *w2, *wis;
-    uint32_t *roff;
-    uint8_t *rbits;
+    uint32_t *slot;     // s-th stored row of the head: offset | width << 16 | row << 24
     __device__ __forceinline__ Stage(uint8_t *base, uint32_t page_region) {
         page = base;
         q = (float *)(base + page_region);
@@ -83,8 +86,7 @@ struct Stage {
         gate = q + 384;
         w2 = q + 512;
         wis = q + 640;
-        roff = (uint32_t *)(q + 768);
-        rbits = (uint8_t *)(q + 896);
+        slot = (uint32_t *)(q + 768);
     }
 };
 
@@ -98,92 +100,75 @@ struct T {   // thread coordinates
     __device__ __forceinline__ int row(int r) const { return 16 * w + r; }
 };
 
-// Duplicated row constants of row i: the (x, x) and (z, z) pairs of a float4.
-__device__ __forceinline__ void row_dup(const float4 *v, int i, uint64_t &xx, uint64_t &zz) {
-    const uint4 q = *(const uint4 *)&v[i];
-    xx = u2pair(q.x, q.y);
-    zz = u2pair(q.z, q.w);
+// Row-pair constants m = 2p, 2p+1 of the warp's band from one 128-bit load.
+__device__ __forceinline__ void row_pairs(const float *v, const T &t, int p, uint64_t &lo, uint64_t &hi) {
+    const uint4 q = *(const uint4 *)&v[t.row(4 * p)];
+    lo = u2pair(q.x, q.y);
+    hi = u2pair(q.z, q.w);
 }
-// The lane's two column pairs of a per-column vector.
-__device__ __forceinline__ void col_pairs(const float *v, int l, uint64_t &p0, uint64_t &p1) {
-    const uint4 q = *(const uint4 *)&v[4 * l];
-    p0 = u2pair(q.x, q.y);
-    p1 = u2pair(q.z, q.w);
+__device__ __forceinline__ uint64_t row_pair(const float *v, const T &t, int m) {
+    return *(const uint64_t *)&v[t.row(2 * m)];
+}
+// The lane's 4 columns of a per-column vector as duplicated pairs.
+__device__ __forceinline__ void col_dup(const float *v, int l, uint64_t (&d)[4]) {
+    const float4 q = *(const float4 *)&v[4 * l];
+    d[0] = f2s(q.x);
+    d[1] = f2s(q.y);
+    d[2] = f2s(q.z);
+    d[3] = f2s(q.w);
 }
 __device__ __forceinline__ void cols_to_red(const T &t, float *red, int reg, const float (&v)[4]) {
     *(float4 *)&red[(reg * 8 + t.w) * 128 + 4 * t.l] = make_float4(v[0], v[1], v[2], v[3]);
 }
+// (lo, hi) clamped to +-lim_lo and +-lim_hi.
+__device__ __forceinline__ uint64_t clamp2p(uint64_t v, uint64_t lim) {
+    const float a = f2lo(lim), b = f2hi(lim);
+    return f2(fminf(fmaxf(f2lo(v), -a), a), fminf(fmaxf(f2hi(v), -b), b));
+}
 
-// Row widths of the warp's band, one byte each in four registers.
-struct Widths {
-    uint32_t w[4];
-    __device__ __forceinline__ Widths(const uint8_t *rbits, int band) {
-        const uint4 q = *(const uint4 *)&rbits[16 * band];
-        w[0] = q.x; w[1] = q.y; w[2] = q.z; w[3] = q.w;
-    }
-    __device__ __forceinline__ int operator[](int r) const { return (w[r >> 2] >> (8 * (r & 3))) & 0xFF; }
-};
-
-// The lane's 4 codes of a row of width B (B < 8), right-aligned in one word.
-template <int B>
-__device__ __forceinline__ uint32_t lane_codes(const uint8_t *row, int l) {
-    if (B == 2) return row[l];
-    if (B == 4) return ((const uint16_t *)row)[l];
-    // B == 6: bytes 3l..3l+2 of the row (the next word may lie past the row;
-    // it stays inside the stage and its bits are masked off)
+// The lane's 4b-bit code segment of a row of width b (columns 4l..4l+3),
+// right-aligned. The second word may lie past the row; it stays inside the
+// stage and its bits beyond the segment are masked off by the callers.
+__device__ __forceinline__ uint32_t lane_segment(const uint8_t *row, int b, int l) {
     const uint32_t *wp = (const uint32_t *)row;
-    const int byte = 3 * l;
-    return __funnelshift_r(wp[byte >> 2], wp[(byte >> 2) + 1], 8 * (byte & 3)) & 0xFFFFFFu;
+    const int bit = 4 * l * b;
+    return __funnelshift_r(wp[bit >> 5], wp[(bit >> 5) + 1], bit & 31);
 }
 
-// Decode the lane's 4 codes of one integer row into (c q) pairs: each code is
-// dropped into the zero mantissa bits of 1.5*2^23 (one logic op), the offset
-// 1.5*2^23 + 2^(B-1) comes off exactly and c_j q_ij is exact in fp32.
-template <int B>
-__device__ __forceinline__ void decode_row(const uint8_t *row, int l, uint64_t c01, uint64_t c23,
-                                           uint64_t &x0, uint64_t &x1) {
-    uint32_t f0, f1, f2, f3;
-    if (B == 8) {
-        const uint32_t w = ((const uint32_t *)row)[l];
-        f0 = __byte_perm(w, kMagicBits, 0x7650);
-        f1 = __byte_perm(w, kMagicBits, 0x7651);
-        f2 = __byte_perm(w, kMagicBits, 0x7652);
-        f3 = __byte_perm(w, kMagicBits, 0x7653);
-    } else {
-        constexpr uint32_t mask = (1u << B) - 1u;
-        const uint32_t x = lane_codes<B>(row, l);
-        f0 = and_or(x, mask, kMagicBits);
-        f1 = and_or(x >> B, mask, kMagicBits);
-        f2 = and_or(x >> (2 * B), mask, kMagicBits);
-        f3 = and_or(x >> (3 * B), mask, kMagicBits);
-    }
-    const uint64_t off = f2s(-(kMagic + (float)(1 << (B - 1))));
-    x0 = fmul2(fadd2(u2pair(f0, f1), off), c01);
-    x1 = fmul2(fadd2(u2pair(f2, f3), off), c23);
-}
-
-// Pack the lane's 4 codes (float bit patterns 0x4B400000 | u) of a row of
-// width B into the row: the known high bits are summed and subtracted once.
-template <int B>
-__device__ __forceinline__ void store_row(uint8_t *row, int l, uint32_t f0, uint32_t f1, uint32_t f2,
-                                          uint32_t f3) {
-    if (B == 8) {
-        const uint32_t lo = __byte_perm(f0, f1, 0x0040), hi = __byte_perm(f2, f3, 0x0040);
-        ((uint32_t *)row)[l] = __byte_perm(lo, hi, 0x5410);
-        return;
-    }
-    constexpr uint32_t K = kMagicBits + (kMagicBits << B) + (kMagicBits << (2 * B)) + (kMagicBits << (3 * B));
-    const uint32_t v = f0 + (f1 << B) + (f2 << (2 * B)) + (f3 << (3 * B)) - K;   // 4B bits
-    if (B == 2) {
-        row[l] = (uint8_t)v;
-    } else if (B == 4) {
+// Write the lane's 4b-bit segment v (b in {2, 4, 6, 8}) into the row.
+__device__ __forceinline__ void store_segment(uint8_t *row, int b, int l, uint32_t v) {
+    if (b == 8) {
+        ((uint32_t *)row)[l] = v;
+    } else if (b == 4) {
         ((uint16_t *)row)[l] = (uint16_t)v;
+    } else if (b == 2) {
+        row[l] = (uint8_t)v;
     } else {
         // 24 bits per lane: lanes 4g..4g+2 each store one of the words 3g..3g+2
         const uint32_t nb = __shfl_down_sync(0xffffffffu, v, 1);
         const int j = l & 3;
         if (j < 3) ((uint32_t *)row)[3 * (l >> 2) + j] = (v >> (8 * j)) | (nb << (24 - 8 * j));
     }
+}
+
+// Sum over the 4 codes of a lane segment of (0x4B400000 << k b): what the
+// packing adds besides the codes.
+__device__ __forceinline__ uint32_t pack_bias4(int b) {
+    return kMagicBits + (kMagicBits << b) + (kMagicBits << (2 * b)) + (kMagicBits << (3 * b));
+}
+
+// FP16 pivot rows (rare): kept out of line so the unrolled tile loops stay small.
+__device__ __noinline__ float4 pivot_values(const uint8_t *row, int l) {
+    const uint2 p = ((const uint2 *)row)[l];
+    return make_float4(f16_val((uint16_t)(p.x & 0xFFFFu)), f16_val((uint16_t)(p.x >> 16)),
+                       f16_val((uint16_t)(p.y & 0xFFFFu)), f16_val((uint16_t)(p.y >> 16)));
+}
+__device__ __noinline__ void store_pivot(uint8_t *row, int l, float a, float4 z) {
+    const uint32_t w0 = (uint32_t)f16_bits(f16_round_sat(a * z.x)) |
+                        ((uint32_t)f16_bits(f16_round_sat(a * z.y)) << 16);
+    const uint32_t w1 = (uint32_t)f16_bits(f16_round_sat(a * z.z)) |
+                        ((uint32_t)f16_bits(f16_round_sat(a * z.w)) << 16);
+    ((uint2 *)row)[l] = make_uint2(w0, w1);
 }
 
 // ------------------------------------------------------------------ decode
@@ -215,90 +200,98 @@ __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h,
     bulk_load(st.gate, a.gate + ((size_t)b * a.Hv + h) * 128, 512, bar);
     bulk_load(st.w2, a.tab.w2 + (size_t)h * 128, 512, bar);
     bulk_load(st.wis, a.tab.wis + (size_t)h * 128, 512, bar);
-    bulk_load(st.roff, a.tab.row_off + (size_t)h * 128, 512, bar);
-    bulk_load(st.rbits, a.tab.row_bits + (size_t)h * 128, 128, bar);
+    bulk_load(st.slot, a.tab.row_slot + (size_t)h * 128, 512, bar);
 }
 
-// Decode of one row r of the thread's band at its width.
-__device__ __forceinline__ void load_row(const T &t, const Stage &st, int B, int r, uint64_t c01,
-                                         uint64_t c23, uint64_t &x0, uint64_t &x1) {
-    const uint8_t *row = st.page + st.roff[t.row(r)];
-    switch (B) {
-    case 2: decode_row<2>(row, t.l, c01, c23, x0, x1); break;
-    case 4: decode_row<4>(row, t.l, c01, c23, x0, x1); break;
-    case 6: decode_row<6>(row, t.l, c01, c23, x0, x1); break;
-    case 8: decode_row<8>(row, t.l, c01, c23, x0, x1); break;
-    default: {
-        const uint2 v = ((const uint2 *)row)[t.l];
-        x0 = f2(f16_val((uint16_t)(v.x & 0xFFFFu)), f16_val((uint16_t)(v.x >> 16)));
-        x1 = f2(f16_val((uint16_t)(v.y & 0xFFFFu)), f16_val((uint16_t)(v.y >> 16)));
-    } break;
+// Z of row pair m (columns 4l..4l+3): c_j q_ij (exact) for integer rows, the
+// FP16 value for pivot rows.
+__device__ __forceinline__ void load_pair(const T &t, const Smem &S, const uint8_t *page, int m,
+                                          const uint64_t (&cd)[4], uint64_t (&x)[4]) {
+    const uint4 inf = *(const uint4 *)&S.rInfo[t.row(2 * m)];
+    const int b0 = (int)((inf.x >> 16) & 0xFFu), b1 = (int)((inf.z >> 16) & 0xFFu);
+    const uint8_t *r0 = page + (inf.x & 0xFFFFu), *r1 = page + (inf.z & 0xFFFFu);
+    float v[2][4];
+#pragma unroll
+    for (int h = 0; h < 2; h++) {
+        const int b = h ? b1 : b0;
+        const uint8_t *row = h ? r1 : r0;
+        if (b == kPivot) {
+            const float4 p = pivot_values(row, t.l);
+            v[h][0] = p.x;
+            v[h][1] = p.y;
+            v[h][2] = p.z;
+            v[h][3] = p.w;
+        } else {
+            const uint32_t s = lane_segment(row, b, t.l), k = (1u << b) - 1u;
+            const float off = S.rOff[t.row(2 * m + h)];
+#pragma unroll
+            for (int c = 0; c < 4; c++)
+                v[h][c] = __fmul_rn(__uint_as_float(and_or(s >> (c * b), k, kMagicBits)) + off,
+                                    f2lo(cd[c]));
+        }
     }
+#pragma unroll
+    for (int c = 0; c < 4; c++) x[c] = f2(v[0][c], v[1][c]);
 }
 
-// Final codes of one row: q = rne(X' / c_j) (clamped to +-qmax when CLIP), or
-// fp16(a Z) for a pivot row.
+// Final codes of row pair m: q = rne(X' / c_j) (clamped to +-qmax when CLIP),
+// or fp16(a Z) for a pivot row, written into the page.
 template <bool CLIP>
-__device__ __forceinline__ void store_final(const T &t, const Smem &S, const Stage &st, int B, int r,
-                                            uint64_t x0, uint64_t x1, uint64_t g01, uint64_t g23) {
-    const int i = t.row(r);
-    uint8_t *row = st.page + st.roff[i];
-    if (B == kPivot) {
-        const float a = S.rowQ[i].z;
-        const uint32_t w0 = (uint32_t)f16_bits(f16_round_sat(a * f2lo(x0))) |
-                            ((uint32_t)f16_bits(f16_round_sat(a * f2hi(x0))) << 16);
-        const uint32_t w1 = (uint32_t)f16_bits(f16_round_sat(a * f2lo(x1))) |
-                            ((uint32_t)f16_bits(f16_round_sat(a * f2hi(x1))) << 16);
-        ((uint2 *)row)[t.l] = make_uint2(w0, w1);
-        return;
+__device__ __forceinline__ void store_pair(const T &t, const Smem &S, uint8_t *page, int m,
+                                           const uint64_t (&x)[4], const uint64_t (&gd)[4]) {
+    const uint4 inf = *(const uint4 *)&S.rInfo[t.row(2 * m)];
+    const int b0 = (int)((inf.x >> 16) & 0xFFu), b1 = (int)((inf.z >> 16) & 0xFFu);
+    uint8_t *r0 = page + (inf.x & 0xFFFFu), *r1 = page + (inf.z & 0xFFFFu);
+    const uint64_t mb = row_pair(S.rMb, t, m);
+    const uint64_t qm = CLIP ? row_pair(S.rQm, t, m) : 0;
+    uint32_t f[2][4];
+#pragma unroll
+    for (int c = 0; c < 4; c++) {
+        uint64_t tq = fmul2(x[c], gd[c]);
+        if (CLIP) tq = clamp2p(tq, qm);
+        const uint64_t uu = fadd2(tq, mb);              // bits: 0x4B400000 | (q + 2^(b-1))
+        f[0][c] = (uint32_t)uu;
+        f[1][c] = (uint32_t)(uu >> 32);
     }
-    uint64_t t0 = fmul2(x0, g01), t1 = fmul2(x1, g23);
-    if (CLIP) {
-        const float qm = S.rowM[i].z;
-        t0 = clamp2(t0, qm);
-        t1 = clamp2(t1, qm);
-    }
-    const uint64_t mb = f2s(kMagic + (float)(1 << (B - 1)));
-    const uint64_t u0 = fadd2(t0, mb), u1 = fadd2(t1, mb);   // bits: 0x4B400000 | (q + 2^(B-1))
-    const uint32_t f0 = (uint32_t)u0, f1 = (uint32_t)(u0 >> 32), f2v = (uint32_t)u1, f3 = (uint32_t)(u1 >> 32);
-    switch (B) {
-    case 2: store_row<2>(row, t.l, f0, f1, f2v, f3); break;
-    case 4: store_row<4>(row, t.l, f0, f1, f2v, f3); break;
-    case 6: store_row<6>(row, t.l, f0, f1, f2v, f3); break;
-    default: store_row<8>(row, t.l, f0, f1, f2v, f3); break;
+#pragma unroll
+    for (int h = 0; h < 2; h++) {
+        const int b = h ? b1 : b0;
+        uint8_t *row = h ? r1 : r0;
+        if (b == kPivot) {
+            store_pivot(row, t.l, S.rA[t.row(2 * m + h)],
+                        make_float4(h ? f2hi(x[0]) : f2lo(x[0]), h ? f2hi(x[1]) : f2lo(x[1]),
+                                    h ? f2hi(x[2]) : f2lo(x[2]), h ? f2hi(x[3]) : f2lo(x[3])));
+        } else {
+            const uint32_t K = h ? inf.w : inf.y;
+            const uint32_t v = f[h][0] + (f[h][1] << b) + (f[h][2] << (2 * b)) + (f[h][3] << (3 * b)) - K;
+            store_segment(row, b, t.l, v);
+        }
     }
 }
 
 template <bool CLIP>
-__device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_t (&x2)[16][2], uint64_t g01,
-                                        uint64_t g23, uint64_t (&n)[2], uint64_t (&d)[2]) {
+__device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_t (&x2)[8][4],
+                                        const uint64_t (&g)[4], uint64_t (&n)[4], uint64_t (&d)[4]) {
     const uint64_t M2 = f2s(kMagic), nM2 = f2s(-kMagic);
 #pragma unroll
-    for (int r = 0; r < 16; r++) {
-        uint64_t rho, al;
-        row_dup(S.rowF, t.row(r), rho, al);
-        uint64_t q0 = fadd2(fadd2(fmul2(x2[r][0], g01), M2), nM2);
-        uint64_t q1 = fadd2(fadd2(fmul2(x2[r][1], g23), M2), nM2);
-        if (CLIP) {
-            const float qm = S.rowM[t.row(r)].z;
-            q0 = clamp2(q0, qm);
-            q1 = clamp2(q1, qm);
-        }
-        const uint64_t a0 = fmul2(al, q0), a1 = fmul2(al, q1);
-        n[0] = ffma2(a0, x2[r][0], n[0]);
-        n[1] = ffma2(a1, x2[r][1], n[1]);
-        d[0] = ffma2(a0, q0, d[0]);
-        d[1] = ffma2(a1, q1, d[1]);
-    }
-}
-
-template <bool CLIP>
-__device__ __forceinline__ void final_codes(const T &t, const Smem &S, const Stage &st, const Widths &wd,
-                                            const uint64_t (&x2)[16][2]) {
-    uint64_t g01, g23;
-    col_pairs(S.colG, t.l, g01, g23);
+    for (int p = 0; p < 4; p++) {
+        uint64_t alo, ahi, qlo = 0, qhi = 0;
+        row_pairs(S.rAl, t, p, alo, ahi);
+        if (CLIP) row_pairs(S.rQm, t, p, qlo, qhi);
 #pragma unroll
-    for (int r = 0; r < 16; r++) store_final<CLIP>(t, S, st, wd[r], r, x2[r][0], x2[r][1], g01, g23);
+        for (int h = 0; h < 2; h++) {
+            const int m = 2 * p + h;
+            const uint64_t al = h ? ahi : alo;
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                uint64_t q = fadd2(fadd2(fmul2(x2[m][c], g[c]), M2), nM2);
+                if (CLIP) q = clamp2p(q, h ? qhi : qlo);
+                const uint64_t aq = fmul2(al, q);
+                n[c] = ffma2(aq, x2[m][c], n[c]);
+                d[c] = ffma2(aq, q, d[c]);
+            }
+        }
+    }
 }
 
 // One decode step of one row-unit head page staged in shared memory
@@ -311,49 +304,60 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     uint16_t *page_c = (uint16_t *)(st.page + 256);
     // Row constants of the warp's band (warp-local).
     if (t.l < 16) {
-        const int i = t.row(t.l);
-        const int b = st.rbits[i];
+        const int sl = t.row(t.l);                         // stored slot; i = its key row
+        const uint32_t info = st.slot[sl];
+        const int b = (int)((info >> 16) & 0xFFu), i = (int)(info >> 24);
         const float dg = st.gate[i];
-        float a = dg, mu = 0.f, qm = 0.f;
+        float a = dg, mu = 0.f, qm = 0.f, mb = 0.f;
+        uint32_t K = 0;
         if (b != kPivot) {
             a = dg * (f16_val(page_r[i]) * (float)(1 << (8 - b)));
             qm = (float)((1 << (b - 1)) - 1);
             mu = __frcp_rn(qm);
+            mb = kMagic + (float)(1 << (b - 1));
+            K = pack_bias4(b);
         }
         a = fmaxf(a, 1e-30f);
-        const float ki = st.k[i], kap = ki * a, bkp = __fdividef(beta * ki, a), qa = st.q[i] * a;
-        S.rowK[i] = make_float4(kap, kap, bkp, bkp);
-        S.rowQ[i] = make_float4(qa, qa, a, a);
-        S.rowM[i] = make_float4(mu, mu, qm, qm);
+        const float ki = st.k[i];
+        S.rKap[sl] = ki * a;
+        S.rBkp[sl] = __fdividef(beta * ki, a);
+        S.rQa[sl] = st.q[i] * a;
+        S.rA[sl] = a;
+        S.rMu[sl] = mu;
+        S.rQm[sl] = qm;
+        S.rOff[sl] = -mb;
+        S.rMb[sl] = mb;
+        S.rInfo[sl] = make_uint2(info, K);
     }
     if (t.tid < 128) S.colM[t.tid] = 0u;
-    // Step 1: Z = c_j q_ij (exact) or the FP16 value.
-    uint64_t x2[16][2];
-    {
-        const uint2 cb = ((const uint2 *)page_c)[t.l];
-        const uint64_t c01 = f2(f16_val((uint16_t)(cb.x & 0xFFFFu)), f16_val((uint16_t)(cb.x >> 16)));
-        const uint64_t c23 = f2(f16_val((uint16_t)(cb.y & 0xFFFFu)), f16_val((uint16_t)(cb.y >> 16)));
-#pragma unroll
-        const Widths wd(st.rbits, t.w);
-#pragma unroll
-        for (int r = 0; r < 16; r++) load_row(t, st, wd[r], r, c01, c23, x2[r][0], x2[r][1]);
-    }
     __syncwarp();
+    // Step 1: Z = c_j q_ij (exact) or the FP16 value.
+    uint64_t x2[8][4];
+    {
+        uint64_t cd[4];
+        const uint2 cb = ((const uint2 *)page_c)[t.l];
+        cd[0] = f2s(f16_val((uint16_t)(cb.x & 0xFFFFu)));
+        cd[1] = f2s(f16_val((uint16_t)(cb.x >> 16)));
+        cd[2] = f2s(f16_val((uint16_t)(cb.y & 0xFFFFu)));
+        cd[3] = f2s(f16_val((uint16_t)(cb.y >> 16)));
+#pragma unroll
+        for (int m = 0; m < 8; m++) load_pair(t, S, st.page, m, cd, x2[m]);
+    }
     // Step 2a: retrieval u_j = sum_i k_i a_i Z_ij.
     {
-        uint64_t ua[2] = {0, 0}, ub[2] = {0, 0};
+        uint64_t ua[4] = {0, 0, 0, 0}, ub[4] = {0, 0, 0, 0};
 #pragma unroll
-        for (int r = 0; r < 16; r += 2) {
-            uint64_t k0, k1, z;
-            row_dup(S.rowK, t.row(r), k0, z);
-            row_dup(S.rowK, t.row(r + 1), k1, z);
-            ua[0] = ffma2(k0, x2[r][0], ua[0]);
-            ua[1] = ffma2(k0, x2[r][1], ua[1]);
-            ub[0] = ffma2(k1, x2[r + 1][0], ub[0]);
-            ub[1] = ffma2(k1, x2[r + 1][1], ub[1]);
+        for (int p = 0; p < 4; p++) {
+            uint64_t klo, khi;
+            row_pairs(S.rKap, t, p, klo, khi);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                ua[c] = ffma2(klo, x2[2 * p][c], ua[c]);
+                ub[c] = ffma2(khi, x2[2 * p + 1][c], ub[c]);
+            }
         }
-        const uint64_t s0 = fadd2(ua[0], ub[0]), s1 = fadd2(ua[1], ub[1]);
-        const float v[4] = {f2lo(s0), f2hi(s0), f2lo(s1), f2hi(s1)};
+        const float v[4] = {pair_sum(fadd2(ua[0], ub[0])), pair_sum(fadd2(ua[1], ub[1])),
+                            pair_sum(fadd2(ua[2], ub[2])), pair_sum(fadd2(ua[3], ub[3]))};
         cols_to_red(t, S.red, 0, v);
     }
     if (__syncthreads_or(!ok)) return false;
@@ -368,49 +372,54 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     // Step 2b-3: Z += (beta k_i / a_i) delta_j; readout partials q_i a_i Z_ij.
     float rs[16];
     {
-        uint64_t d01, d23;
-        col_pairs(S.colD, t.l, d01, d23);
-        uint64_t ya[2] = {0, 0}, yb[2] = {0, 0};
+        uint64_t dl[4];
+        col_dup(S.colD, t.l, dl);
+        uint64_t ya[4] = {0, 0, 0, 0}, yb[4] = {0, 0, 0, 0};
 #pragma unroll
-        for (int r = 0; r < 16; r++) {
-            uint64_t z, bk, qa;
-            row_dup(S.rowK, t.row(r), z, bk);
-            row_dup(S.rowQ, t.row(r), qa, z);
-            x2[r][0] = ffma2(bk, d01, x2[r][0]);
-            x2[r][1] = ffma2(bk, d23, x2[r][1]);
-            if (r & 1) {
-                yb[0] = ffma2(qa, x2[r][0], yb[0]);
-                yb[1] = ffma2(qa, x2[r][1], yb[1]);
-            } else {
-                ya[0] = ffma2(qa, x2[r][0], ya[0]);
-                ya[1] = ffma2(qa, x2[r][1], ya[1]);
+        for (int p = 0; p < 4; p++) {
+            uint64_t blo, bhi, qlo, qhi;
+            row_pairs(S.rBkp, t, p, blo, bhi);
+            row_pairs(S.rQa, t, p, qlo, qhi);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                x2[2 * p][c] = ffma2(blo, dl[c], x2[2 * p][c]);
+                x2[2 * p + 1][c] = ffma2(bhi, dl[c], x2[2 * p + 1][c]);
+                ya[c] = ffma2(qlo, x2[2 * p][c], ya[c]);
+                yb[c] = ffma2(qhi, x2[2 * p + 1][c], yb[c]);
             }
-            rs[r] = (fabsf(f2lo(x2[r][0])) + fabsf(f2hi(x2[r][0]))) +
-                    (fabsf(f2lo(x2[r][1])) + fabsf(f2hi(x2[r][1])));
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                const uint64_t(&xm)[4] = x2[2 * p + h];
+                rs[4 * p + 2 * h] = (fabsf(f2lo(xm[0])) + fabsf(f2lo(xm[1]))) +
+                                    (fabsf(f2lo(xm[2])) + fabsf(f2lo(xm[3])));
+                rs[4 * p + 2 * h + 1] = (fabsf(f2hi(xm[0])) + fabsf(f2hi(xm[1]))) +
+                                        (fabsf(f2hi(xm[2])) + fabsf(f2hi(xm[3])));
+            }
         }
-        const uint64_t s0 = fadd2(ya[0], yb[0]), s1 = fadd2(ya[1], yb[1]);
-        const float v[4] = {f2lo(s0), f2hi(s0), f2lo(s1), f2hi(s1)};
+        const float v[4] = {pair_sum(fadd2(ya[0], yb[0])), pair_sum(fadd2(ya[1], yb[1])),
+                            pair_sum(fadd2(ya[2], yb[2])), pair_sum(fadd2(ya[3], yb[3]))};
         cols_to_red(t, S.red, 2, v);
     }
     // Step 4: row factors r_i = m_i^(1/2) w_i^(-1/2) of the integer rows.
     {
         int rr;
         const float sz = warp_row_sums(rs, t.l, rr);
-        const int i = t.row(rr);
-        const int b = st.rbits[i];
+        const int sl = t.row(rr);
         if ((t.l & 1) == 0) {
+            const uint32_t info = S.rInfo[sl].x;
+            const int b = (int)((info >> 16) & 0xFFu), i = (int)(info >> 24);
             if (b == kPivot) {
-                S.rowF[i] = make_float4(1.f, 1.f, 0.f, 0.f);
+                S.rRho[sl] = 1.f;
+                S.rAl[sl] = 0.f;
                 page_r[i] = 0;
             } else {
-                const float a = S.rowQ[i].z;
+                const float a = S.rA[sl];
                 const float m = (a * sz) * (1.0f / 128.0f);
                 const float rf = __half2float(__float2half_rn(
                     fminf(fmaxf(__fmul_rn(sqrtf(m), st.wis[i]), kF16Min), kF16Max)));
                 const float rz = rf * (float)(1 << (8 - b));          // r_i zs_i, exact
-                const float rho_a = __frcp_rn(rz) * a;                // X' = rho_i X = (rho_i a_i) Z
-                const float al = st.w2[i] * (rz * rz);                // w_i^2 (r_i zs_i)^2
-                S.rowF[i] = make_float4(rho_a, rho_a, al, al);
+                S.rRho[sl] = __frcp_rn(rz) * a;                       // X' = rho_i X = (rho_i a_i) Z
+                S.rAl[sl] = st.w2[i] * (rz * rz);                     // w_i^2 (r_i zs_i)^2
                 page_r[i] = f16_bits(rf);
             }
         }
@@ -421,19 +430,17 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     {
         float cm[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int r = 0; r < 16; r += 2) {
-            uint64_t rho0, rho1, mu0, mu1, z;
-            row_dup(S.rowF, t.row(r), rho0, z);
-            row_dup(S.rowF, t.row(r + 1), rho1, z);
-            row_dup(S.rowM, t.row(r), mu0, z);
-            row_dup(S.rowM, t.row(r + 1), mu1, z);
+        for (int p = 0; p < 4; p++) {
+            uint64_t rlo, rhi, mlo, mhi;
+            row_pairs(S.rRho, t, p, rlo, rhi);
+            row_pairs(S.rMu, t, p, mlo, mhi);
 #pragma unroll
-            for (int p = 0; p < 2; p++) {
-                x2[r][p] = fmul2(x2[r][p], rho0);
-                x2[r + 1][p] = fmul2(x2[r + 1][p], rho1);
-                const uint64_t m0 = fmul2(x2[r][p], mu0), m1 = fmul2(x2[r + 1][p], mu1);
-                cm[2 * p] = fmax3(cm[2 * p], fabsf(f2lo(m0)), fabsf(f2lo(m1)));
-                cm[2 * p + 1] = fmax3(cm[2 * p + 1], fabsf(f2hi(m0)), fabsf(f2hi(m1)));
+            for (int c = 0; c < 4; c++) {
+                x2[2 * p][c] = fmul2(x2[2 * p][c], rlo);
+                x2[2 * p + 1][c] = fmul2(x2[2 * p + 1][c], rhi);
+                const uint64_t e0 = fmul2(x2[2 * p][c], mlo), e1 = fmul2(x2[2 * p + 1][c], mhi);
+                cm[c] = fmax3(cm[c], fabsf(f2lo(e0)), fabsf(f2hi(e0)));
+                cm[c] = fmax3(cm[c], fabsf(f2lo(e1)), fabsf(f2hi(e1)));
             }
         }
 #pragma unroll
@@ -462,14 +469,14 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     // Step 5: fixed-code least-squares updates of c over the integer rows.
     const bool clip0 = S.flags[1] != 0;
     for (int it = 0; it < fit_iters; it++) {
-        uint64_t g01, g23;
-        col_pairs(S.colG, t.l, g01, g23);
-        uint64_t n[2] = {0, 0}, d[2] = {0, 0};
-        if (it > 0 || clip0) ls_sums<true>(t, S, x2, g01, g23, n, d);
-        else ls_sums<false>(t, S, x2, g01, g23, n, d);
+        uint64_t g[4];
+        col_dup(S.colG, t.l, g);
+        uint64_t n[4] = {0, 0, 0, 0}, d[4] = {0, 0, 0, 0};
+        if (it > 0 || clip0) ls_sums<true>(t, S, x2, g, n, d);
+        else ls_sums<false>(t, S, x2, g, n, d);
         {
-            const float vn[4] = {f2lo(n[0]), f2hi(n[0]), f2lo(n[1]), f2hi(n[1])};
-            const float vd[4] = {f2lo(d[0]), f2hi(d[0]), f2lo(d[1]), f2hi(d[1])};
+            const float vn[4] = {pair_sum(n[0]), pair_sum(n[1]), pair_sum(n[2]), pair_sum(n[3])};
+            const float vd[4] = {pair_sum(d[0]), pair_sum(d[1]), pair_sum(d[2]), pair_sum(d[3])};
             cols_to_red(t, S.red, 0, vn);
             cols_to_red(t, S.red, 1, vd);
         }
@@ -500,9 +507,17 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         __syncthreads();
     }
     // Step 6: final codes with the stored scales, written in place.
-    const Widths wd(st.rbits, t.w);
-    if (S.flags[2]) final_codes<true>(t, S, st, wd, x2);
-    else final_codes<false>(t, S, st, wd, x2);
+    {
+        uint64_t gd[4];
+        col_dup(S.colG, t.l, gd);
+        if (S.flags[2]) {
+#pragma unroll
+            for (int m = 0; m < 8; m++) store_pair<true>(t, S, st.page, m, x2[m], gd);
+        } else {
+#pragma unroll
+            for (int m = 0; m < 8; m++) store_pair<false>(t, S, st.page, m, x2[m], gd);
+        }
+    }
     return true;
 }
 
@@ -539,15 +554,6 @@ __global__ void __launch_bounds__(kThreads, 2) decode_rows_kernel(DecodeArgs a) 
 
 }  // namespace rk
 
-static int sm_count_rows() {
-    static int n[64];
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 0 || dev >= 64) return 1;
-    if (!n[dev]) cudaDeviceGetAttribute(&n[dev], cudaDevAttrMultiProcessorCount, dev);
-    return n[dev] > 0 ? n[dev] : 1;
-}
-
 stepq_status launch_decode_rows(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
                                 const int32_t *slots, int B, const float *q, const float *k,
                                 const float *v, const float *beta, const float *gate, float *y,
@@ -580,7 +586,10 @@ stepq_status launch_decode_rows(const stepq_plan *p, int layer, uint8_t *pool, i
     if (cudaFuncSetAttribute((const void *)rk::decode_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              smem) != cudaSuccess)
         return STEPQ_ERR_CUDA;
-    int grid = 2 * sm_count_rows();
+    int dev = 0, sms = 1;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    int grid = 2 * (sms > 0 ? sms : 1);
     if (grid > a.items) grid = a.items;
     rk::decode_rows_kernel<<<grid, kThreads, smem, s>>>(a);
     return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;

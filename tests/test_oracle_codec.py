@@ -112,14 +112,16 @@ def test_bit_layout_with_independent_unpacker(oracle, rng, b):
 
 def test_row_unit_layout_with_independent_unpacker(oracle, rng):
     """Row units: r | c | row i holds its 128 codes (b_i bits, LSB-first), FP16 rows
-    for pivots; rows follow each other in index order."""
+    for pivots; rows are stored by decreasing width, equal widths in index order."""
     X = _state(rng)
     rb = _widths(rng, ROW)
     page = oracle.encode_head(X, ROW, rb, _w(rng))
     assert page.size == 512 + 16 * int(np.sum(rb.astype(np.int64)))
     _, _, codes, piv = oracle.unpack_head(page, ROW, rb)
+    order = sorted(range(D), key=lambda i: (-int(rb[i]), i))
+    assert len(set(rb.tolist())) > 2                # the order is not trivial
     off = 512
-    for i in range(D):
+    for i in order:
         b = int(rb[i])
         row = page[off:off + 16 * b]
         if b == PIV:
