@@ -169,6 +169,24 @@ stepq_status stepq_decode_step(const stepq_plan *plan, int layer, void *pool, in
                                const float *v, const float *beta, const float *gate, float *y,
                                stepq_stream_t stream);
 
+/* Prefill of T tokens on FP32 states (the uncompressed side of the prefill
+ * boundary, App. F: the chunk computation runs on the uncompressed state, which
+ * stepq_quantize_pool then packs once). Evaluates the gated Delta rule
+ * (Eq. delta_update) for every slot and value head over T tokens, 32 tokens at
+ * a time in its chunkwise (WY) form, and writes every token's readout.
+ * states: device fp32 [B][Hv][128][128], read as the state before the first
+ *   token and overwritten with the state after the last (zero for a new
+ *   sequence; stepq_dequantize_pool unpacks a stored one).
+ * q, k: [B][T][Hk][128]; v: [B][T][Hv][128]; beta: [B][T][Hv]; gate:
+ *   [B][T][Hv] (scalar) or [B][T][Hv][128] (channel), values in (0, 1]: the
+ *   product of one chunk's gates must stay above 1e-30.
+ * y: [B][T][Hv][128] out. Only dk, dv, heads and gate_kind of cfg are read;
+ * all buffers 16-byte aligned. */
+stepq_status stepq_prefill_fp32(const stepq_config *cfg, int B, int T, float *states,
+                                const float *q, const float *k, const float *v,
+                                const float *beta, const float *gate, float *y,
+                                stepq_stream_t stream);
+
 /* --------------------------------------------------- comparison kernels (same build)
  * FP32-state decode (the serving default the paper compares against, Sec. 5.1):
  * pool: device fp32 [pool_slots][L][Hv][128][128]; the step updates the layer's

@@ -230,6 +230,20 @@ def stepq_fp32_decode_step(cfg: Config, layer: int, pool, slots, q, k, v, beta, 
                                             _stream(stream)), "stepq_fp32_decode_step")
 
 
+def stepq_prefill_fp32(cfg: Config, states, q, k, v, beta, gate, y, stream=None):
+    """Chunked prefill over T tokens on FP32 states [B][Hv][128][128] (in place);
+    q, k [B][T][Hk][128], v [B][T][Hv][128], beta [B][T][Hv], gate [B][T][Hv]
+    or [B][T][Hv][128], y [B][T][Hv][128] out."""
+    import torch
+    f = torch.float32
+    c = cfg.c()
+    B, T = int(q.shape[0]), int(q.shape[1])
+    check(_lib.lib().stepq_prefill_fp32(C.byref(c), B, T, _dev_ptr(states, f), _dev_ptr(q, f),
+                                        _dev_ptr(k, f), _dev_ptr(v, f), _dev_ptr(beta, f),
+                                        _dev_ptr(gate, f), _dev_ptr(y, f), _stream(stream)),
+          "stepq_prefill_fp32")
+
+
 def stepq_intb_slot_bytes(cfg: Config, bits: int) -> int:
     c = cfg.c()
     return int(_lib.lib().stepq_intb_slot_bytes(C.byref(c), bits))

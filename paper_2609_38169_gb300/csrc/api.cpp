@@ -99,6 +99,19 @@ extern "C" stepq_status stepq_fp32_decode_step(const stepq_config *cfg, int laye
                               (cudaStream_t)stream);
 }
 
+extern "C" stepq_status stepq_prefill_fp32(const stepq_config *cfg, int B, int T, float *states,
+                                           const float *q, const float *k, const float *v,
+                                           const float *beta, const float *gate, float *y,
+                                           stepq_stream_t stream) {
+    stepq_status st = validate_config(cfg, false);
+    if (st != STEPQ_OK) return st;
+    if (B < 0 || T < 0 || (B > 0 && T > 0 && (!states || !v || !y))) return STEPQ_ERR_ARG;
+    if (B == 0 || T == 0) return STEPQ_OK;
+    if (!aligned(states, 16)) return STEPQ_ERR_ALIGN;
+    if ((st = check_inputs(cfg, q, k, v, beta, gate, y)) != STEPQ_OK) return st;
+    return launch_prefill(cfg, q, k, v, beta, gate, B, T, states, y, (cudaStream_t)stream);
+}
+
 extern "C" size_t stepq_intb_slot_bytes(const stepq_config *cfg, int bits) {
     if (validate_config(cfg, false) != STEPQ_OK || (bits != 4 && bits != 8)) return 0;
     size_t page = intb_head_bytes(bits) * cfg->n_value_heads * cfg->n_layers;

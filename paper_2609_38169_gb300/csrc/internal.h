@@ -89,6 +89,10 @@ stepq_status launch_quantize(const stepq_plan *p, int layer, const float *states
 stepq_status launch_dequantize(const stepq_plan *p, int layer, const uint8_t *pool, int pool_slots,
                                const int32_t *slots, int B, float *states, size_t state_stride_b,
                                cudaStream_t s);
+// prefill.cu (chunked FP32-state prefill)
+stepq_status launch_prefill(const stepq_config *cfg, const float *q, const float *k, const float *v,
+                            const float *beta, const float *gate, int B, int T, float *states, float *y,
+                            cudaStream_t s);
 // rows.cu (row units, row-major pages with per-row widths)
 stepq_status launch_decode_rows(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
                                 const int32_t *slots, int B, const float *q, const float *k,

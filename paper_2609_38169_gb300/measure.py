@@ -1,0 +1,126 @@
+"""Measurements of the kernels beside the headline decode step (which bench.py
+times): the row-unit decode step against the FP32-state and INT8 comparison
+kernels on one layer of a channel-gate pool, and the chunked FP32 prefill.
+Each subcommand prints one JSON line; inputs are synthetic (the workload
+generators), resident on the device, and timed with CUDA events after warm-up.
+
+    python -m paper_2609_38169_gb300.measure rows [--slots 1024] [--bits 6]
+    python -m paper_2609_38169_gb300.measure prefill [--slots 128] [--tokens 512]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+from . import api as A, workloads as W
+
+D = 128
+FP32_FMA_PEAK_FLOPS = 128 * 2 * 152 * 2.07e9     # FMA lanes/clk/SM x 2 x SMs x max SM clock
+
+
+def _timeit(fn, n=20, warmup=3):
+    import torch
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(n):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / n * 1e-3          # seconds per call
+
+
+def rows(slots=1024, bits=6):
+    """One layer of the drift workload's shape (32 heads, channel gates) over
+    `slots` slots in a random permutation: STEPQuant row units against the
+    FP32-state and INT8 rowwise kernels on identical inputs."""
+    import torch
+    dev = torch.device("cuda")
+    wl = W.WORKLOADS["drift"].replace(layers=1, batch=slots, pool_slots=slots, nominal_bits=bits,
+                                      candidates=(4, 6, 8) if bits == 6 else (2, 4, 6, 8))
+    cfg = A.Config.from_workload(wl)
+    st = A.calibrate(cfg, wl, dev, seqs=4, steps=64, device_inputs=True)
+    plan = A.stepq_fit_scales(cfg, st.omega, st.mean_log_ret, st.dist, st.pivot)
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    S = torch.randn((slots, 1, wl.hv, D, D), generator=g, device=dev)
+    S *= torch.exp(torch.randn((slots, 1, wl.hv, D, 1), generator=g, device=dev))
+    all_slots = torch.arange(slots, dtype=torch.int32, device=dev)
+    perm = torch.from_numpy(W.slot_permutation(wl)).to(dev)
+    pool = A.alloc_pool(plan, slots, dev)
+    A.stepq_quantize_pool(plan, -1, S, all_slots, pool)
+    q, k, v, beta, gate = W.torch_step_inputs(wl, W.model_params_torch(W.model_params(wl), dev), 0, 0, dev)
+    y = torch.empty((slots, wl.hv, D), device=dev)
+    units = slots * wl.hv
+    vec = 4 * 512 + 512 + 4                                    # q k v gate y beta per head update
+    out = {"metric": "row-unit decode step, one layer", "unit": "head-updates/s",
+           "workload": f"{slots} slots x {wl.hv} heads, channel gates, STEPQuant @{bits}",
+           "kernels": {}}
+    t = _timeit(lambda: A.stepq_decode_step(plan, 0, pool, perm, q, k, v, beta, gate, y))
+    page = plan.slot_stride / wl.hv
+    out["kernels"]["stepq_rows"] = {"us_per_launch": t * 1e6, "value": units / t,
+                                    "algorithmic_gbs": units * (2 * page + vec) / t / 1e9,
+                                    "bits_per_value": 8 * page / (D * D)}
+    ref = S.clone()
+    t = _timeit(lambda: A.stepq_fp32_decode_step(cfg, 0, ref, perm, q, k, v, beta, gate, y))
+    out["kernels"]["fp32_state"] = {"us_per_launch": t * 1e6, "value": units / t,
+                                    "algorithmic_gbs": units * (2 * 4 * D * D + vec) / t / 1e9}
+    sb = A.stepq_intb_slot_bytes(cfg, 8)
+    pi = torch.zeros(slots * sb, dtype=torch.uint8, device=dev)
+    A.stepq_intb_quantize_pool(cfg, 8, -1, S, all_slots, pi)
+    t = _timeit(lambda: A.stepq_intb_decode_step(cfg, 8, 0, pi, perm, q, k, v, beta, gate, y))
+    out["kernels"]["int8_rowwise"] = {"us_per_launch": t * 1e6, "value": units / t,
+                                      "algorithmic_gbs": units * (2 * sb / wl.hv + vec) / t / 1e9}
+    assert A.stepq_device_error() == 0
+    return out
+
+
+def prefill(slots=128, tokens=512, name="gqa"):
+    """Chunked FP32 prefill of `tokens` tokens for `slots` slots of one layer."""
+    import torch
+    dev = torch.device("cuda")
+    wl = W.WORKLOADS[name].replace(batch=slots, pool_slots=slots)
+    cfg = A.Config.from_workload(wl)
+    mp = W.model_params_torch(W.model_params(wl), dev)
+    steps = [W.torch_step_inputs(wl, mp, t, 0, dev) for t in range(tokens)]
+    q, k, v, beta, gate = [torch.stack([s[i] for s in steps], dim=1).contiguous() for i in range(5)]
+    del steps
+    states = torch.zeros((slots, wl.hv, D, D), device=dev)
+    y = torch.empty((slots, tokens, wl.hv, D), device=dev)
+    t = _timeit(lambda: A.stepq_prefill_fp32(cfg, states, q, k, v, beta, gate, y), n=5, warmup=2)
+    head_tokens = slots * tokens * wl.hv
+    C = 32
+    # FMAs of the chunkwise form per head-token: K~S, Q~S and the state update
+    # (3 x 128 x 128), A and Q~K^T (2 x C x 128), the solve and Bm W (1.5 x C x 128)
+    fma = 3 * D * D + 2 * C * D + 1.5 * C * D
+    assert A.stepq_device_error() == 0
+    return {"metric": "chunked FP32 prefill", "unit": "head-tokens/s", "value": head_tokens / t,
+            "tokens_per_s": slots * tokens / t, "ms_per_call": t * 1e3,
+            "workload": f"{name}: {slots} slots x {wl.hv} heads x {tokens} tokens",
+            "roofline": {"bound": "fma", "achieved": 2 * fma * head_tokens / t / 1e12,
+                         "peak": FP32_FMA_PEAK_FLOPS / 1e12, "unit": "TFLOP/s",
+                         "frac": 2 * fma * head_tokens / t / FP32_FMA_PEAK_FLOPS}}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    sub = ap.add_subparsers(dest="what", required=True)
+    r = sub.add_parser("rows")
+    r.add_argument("--slots", type=int, default=1024)
+    r.add_argument("--bits", type=int, default=6, choices=[4, 6])
+    p = sub.add_parser("prefill")
+    p.add_argument("--slots", type=int, default=128)
+    p.add_argument("--tokens", type=int, default=512)
+    p.add_argument("--workload", default="gqa", choices=["gqa", "channel", "pool"])
+    args = ap.parse_args(argv)
+    if args.what == "rows":
+        res = rows(args.slots, args.bits)
+    else:
+        res = prefill(args.slots, args.tokens, args.workload)
+    print(json.dumps(res))
+
+
+if __name__ == "__main__":
+    main()

@@ -123,3 +123,12 @@ def test_drift_variants_and_cli():
     with pytest.raises(SystemExit) as e:
         drift.main(["--help"])
     assert e.value.code == 0
+
+
+def test_measure_cli():
+    """The secondary-measurement module parses its subcommands (no device work)."""
+    from paper_2609_38169_gb300 import measure
+    for argv in (["--help"], ["rows", "--help"], ["prefill", "--help"]):
+        with pytest.raises(SystemExit) as e:
+            measure.main(argv)
+        assert e.value.code == 0
