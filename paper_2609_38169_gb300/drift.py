@@ -33,6 +33,16 @@ VARIANTS = {
     "int8": dict(kind="intb", bits=8),
     "int4": dict(kind="intb", bits=4),
 }
+# Component ablations of Sec. 5.4 that the plan alone expresses: the spatial
+# codec at one uniform width without pivots ("Spatial only"), and the full
+# allocation without its FP16 pivots.
+ABLATIONS = {
+    "spatial6": dict(kind="stepq", nominal_bits=6, candidates=(6,), n_pivots=0),
+    "spatial4": dict(kind="stepq", nominal_bits=4, candidates=(4,), n_pivots=0),
+    "stepq6_nopiv": dict(kind="stepq", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0),
+    "stepq4_nopiv": dict(kind="stepq", nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=0),
+}
+ALL = {**VARIANTS, **ABLATIONS}
 
 
 class _Variant:
@@ -42,7 +52,8 @@ class _Variant:
         self.kind = spec["kind"]
         L = wl.layers
         if self.kind == "stepq":
-            wlv = wl.replace(nominal_bits=spec["nominal_bits"], candidates=spec["candidates"])
+            wlv = wl.replace(nominal_bits=spec["nominal_bits"], candidates=spec["candidates"],
+                             n_pivots=spec.get("n_pivots", wl.n_pivots))
             self.cfg = A.Config.from_workload(wlv)
             st = A.calibrate(self.cfg, wlv, device, device_inputs=True, **calib)
             self.plan = A.stepq_fit_scales(self.cfg, st.omega, st.mean_log_ret, st.dist, st.pivot)
@@ -87,7 +98,7 @@ def run(wl=None, steps=None, every=512, batch=None, variants=tuple(VARIANTS), wa
         for layer in range(L):
             inp = W.torch_step_inputs(wl, mp_dev, t, layer, dev, W.STREAM_WARMUP)
             A.stepq_fp32_decode_step(cfg, layer, ref, slots, *inp, y_ref[layer])
-    vs = [_Variant(n, VARIANTS[n], wl, slots, ref, dev, calib) for n in variants]
+    vs = [_Variant(n, ALL[n], wl, slots, ref, dev, calib) for n in variants]
     ys = torch.empty((len(vs), L, B, Hv, D), dtype=torch.float32, device=dev)
     err_win = torch.zeros(len(vs), dtype=torch.float64, device=dev)
     ref_win = torch.zeros((), dtype=torch.float64, device=dev)
@@ -133,7 +144,8 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=None)
     ap.add_argument("--every", type=int, default=512)
     ap.add_argument("--batch", type=int, default=None)
-    ap.add_argument("--variants", default=",".join(VARIANTS))
+    ap.add_argument("--variants", default=",".join(VARIANTS),
+                    help="comma list from " + ", ".join(ALL))
     ap.add_argument("--out", default=None, help="write the JSON result here")
     args = ap.parse_args(argv)
     res = run(steps=args.steps, every=args.every, batch=args.batch,
