@@ -197,10 +197,24 @@ stepq_status stepq_fp32_decode_step(const stepq_config *cfg, int layer, float *p
                                     const float *k, const float *v, const float *beta,
                                     const float *gate, float *y, stepq_stream_t stream);
 
+/* The exact-read counterpart of stepq_fp32_decode_step used by the feedback
+ * experiment of App. B.4 ("exact-read oracle"): the retrieval reads the
+ * reference states, u = k^T D S_ref with S_ref from read_pool (same layout as
+ * pool, not modified), while the update writes D S + beta k (v - u)^T into
+ * pool. A state error E = S - S_ref then evolves as D E, without the Delta
+ * rule's own correction (Eq. self_correction). */
+stepq_status stepq_fp32_exact_read_step(const stepq_config *cfg, int layer, float *pool,
+                                        const float *read_pool, int pool_slots,
+                                        const int32_t *slots, int B, const float *q,
+                                        const float *k, const float *v, const float *beta,
+                                        const float *gate, float *y, stepq_stream_t stream);
+
 /* Uniform rowwise-absmax INT-b state (App. B.5): per key row an FP16 scale
  * absmax/q_b clamped to [2^-14, 65504], nearest codes in [-q_b, q_b]. Head
  * segment: s[128] fp16 | 128 rows x 16b bytes; segments in (layer, head)
- * order; slot stride = stepq_intb_slot_bytes(). bits: 4 or 8. */
+ * order; slot stride = stepq_intb_slot_bytes(). bits: 4, 6 or 8 (codes
+ * offset-binary, LSB-first along the row); other widths give 0 bytes and
+ * STEPQ_ERR_UNSUPPORTED. */
 size_t stepq_intb_slot_bytes(const stepq_config *cfg, int bits);
 stepq_status stepq_intb_quantize_pool(const stepq_config *cfg, int bits, int layer,
                                       const float *states, const int32_t *slots, int B,

@@ -69,6 +69,8 @@ def _declare(L):
         "or_fp16_decode": (D_, [C.c_uint16]),
         "or_delta_step_f32": (None, [P, P, P, P, F, P, I, P]),
         "or_delta_batch_f32": (None, [I, I, I, I, P, P, P, P, P, P, P]),
+        "or_delta_step_read_f32": (None, [P, P, P, P, P, F, P, I, P]),
+        "or_delta_batch_read_f32": (None, [I, I, I, I, P, P, P, P, P, P, P, P]),
         "or_row_impact": (None, [P, P, F, P, I, P]),
         "or_row_impact_dense": (None, [P, P, F, P, I, P]),
         "or_head_bytes": (C.c_size_t, [I, P]),
@@ -163,6 +165,31 @@ def delta_batch(S, q, k, v, beta, gate):
     y = np.zeros((n, Hv, D), np.float32)
     lib().or_delta_batch_f32(n, Hk, Hv, int(gate.ndim == 3), _p(S), _p(_f32(q)), _p(_f32(k)),
                              _p(_f32(v)), _p(_f32(beta)), _p(gate), _p(y))
+    return y
+
+
+def delta_step_read(S, S_ref, q, k, v, beta, gate):
+    """Exact-read step of one head (App. B.4): the Delta residual reads the
+    reference state, u = k^T D S_ref; returns (S_new, y)."""
+    S = _f32(S).copy()
+    gate = _f32(np.atleast_1d(gate))
+    y = np.zeros(D, np.float32)
+    lib().or_delta_step_read_f32(_p(S), _p(_f32(S_ref)), _p(_f32(q)), _p(_f32(k)), _p(_f32(v)),
+                                 float(beta), _p(gate), int(gate.size == D), _p(y))
+    return S, y
+
+
+def delta_batch_read(S, S_ref, q, k, v, beta, gate):
+    """In-place exact-read step of S [n][Hv][128][128] reading S_ref (same
+    shape); returns y [n][Hv][128]."""
+    assert S.dtype == np.float32 and S.flags["C_CONTIGUOUS"] and S_ref.shape == S.shape
+    n, Hv = S.shape[:2]
+    Hk = q.shape[1]
+    gate = _f32(gate)
+    y = np.zeros((n, Hv, D), np.float32)
+    lib().or_delta_batch_read_f32(n, Hk, Hv, int(gate.ndim == 3), _p(S), _p(_f32(S_ref)),
+                                  _p(_f32(q)), _p(_f32(k)), _p(_f32(v)), _p(_f32(beta)),
+                                  _p(gate), _p(y))
     return y
 
 

@@ -51,6 +51,12 @@ void or_delta_step_f32(float *S, const float *q, const float *k, const float *v,
 void or_delta_batch_f32(int n, int Hk, int Hv, int gate_per_row, float *S,
                         const float *q, const float *k, const float *v,
                         const float *beta, const float *gate, float *y);
+void or_delta_step_read_f32(float *S, const float *Sref, const float *q, const float *k,
+                            const float *v, float beta, const float *gate, int gate_per_row,
+                            float *y);
+void or_delta_batch_read_f32(int n, int Hk, int Hv, int gate_per_row, float *S, const float *Sref,
+                             const float *q, const float *k, const float *v,
+                             const float *beta, const float *gate, float *y);
 void or_row_impact(const float *q, const float *k, float beta, const float *gate,
                    int gate_per_row, double *g);
 void or_row_impact_dense(const float *q, const float *k, float beta, const float *gate,

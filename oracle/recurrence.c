@@ -64,6 +64,59 @@ void or_delta_batch_f32(int n, int Hk, int Hv, int gate_per_row, float *S,
         }
 }
 
+/* The exact-read step of the feedback experiment (App. B.4): only the state
+ * inside the Delta residual is replaced by the reference state S_ref,
+ *   S_t = D_t S_{t-1} + beta_t k_t (v_t^T - k_t^T D_t S_ref_{t-1}),
+ * so that S_t - S_ref_t = D_t (S_{t-1} - S_ref_{t-1}). S is updated in place;
+ * S_ref is only read; y = S_t^T q_t. */
+void or_delta_step_read_f32(float *S, const float *Sref, const float *q, const float *k,
+                            const float *v, float beta, const float *gate, int gate_per_row,
+                            float *y)
+{
+    double u[OR_D];
+    for (int j = 0; j < OR_D; j++) {                              /* k^T D S_ref */
+        double acc = 0.0;
+        for (int i = 0; i < OR_D; i++) {
+            double d = gate_per_row ? gate[i] : gate[0];
+            acc += (double)k[i] * (d * (double)Sref[i * OR_D + j]);
+        }
+        u[j] = acc;
+    }
+    for (int i = 0; i < OR_D; i++) {
+        double d = gate_per_row ? gate[i] : gate[0];
+        for (int j = 0; j < OR_D; j++)
+            S[i * OR_D + j] = (float)(d * (double)S[i * OR_D + j] +
+                                      (double)beta * (double)k[i] * ((double)v[j] - u[j]));
+    }
+    for (int j = 0; j < OR_D; j++) {
+        double acc = 0.0;
+        for (int i = 0; i < OR_D; i++)
+            acc += (double)q[i] * (double)S[i * OR_D + j];
+        y[j] = (float)acc;
+    }
+}
+
+/* Batch form of or_delta_step_read_f32 with the layout of or_delta_batch_f32;
+ * Sref has the layout of S. */
+void or_delta_batch_read_f32(int n, int Hk, int Hv, int gate_per_row, float *S, const float *Sref,
+                             const float *q, const float *k, const float *v,
+                             const float *beta, const float *gate, float *y)
+{
+    int grp = Hv / Hk;
+#pragma omp parallel for collapse(2) schedule(dynamic)
+    for (int b = 0; b < n; b++)
+        for (int h = 0; h < Hv; h++) {
+            int hk = h / grp;
+            size_t o = ((size_t)b * Hv + h) * OR_N;
+            const float *g = gate_per_row ? gate + ((size_t)b * Hv + h) * OR_D
+                                          : gate + (size_t)b * Hv + h;
+            or_delta_step_read_f32(S + o, Sref + o, q + ((size_t)b * Hk + hk) * OR_D,
+                                   k + ((size_t)b * Hk + hk) * OR_D,
+                                   v + ((size_t)b * Hv + h) * OR_D, beta[(size_t)b * Hv + h], g,
+                                   gate_per_row, y + ((size_t)b * Hv + h) * OR_D);
+        }
+}
+
 /* Row-impact vector g_t = A_t^T q_t (Sec. 4.1), closed form of Eq.
  * kda_sensitivity: g_i = d_i [q_i - beta k_i (k^T q)]. */
 void or_row_impact(const float *q, const float *k, float beta, const float *gate,

@@ -42,6 +42,7 @@ SIGNATURES = {
     "stepq_decode_step": (I, [P, I, P, I, P, I, P, P, P, P, P, P, P]),
     "stepq_fp32_decode_step": (I, [CFG, I, P, I, P, I, P, P, P, P, P, P, P]),
     "stepq_prefill_fp32": (I, [CFG, I, I, P, P, P, P, P, P, P, P]),
+    "stepq_fp32_exact_read_step": (I, [CFG, I, P, P, I, P, I, P, P, P, P, P, P, P]),
     "stepq_intb_slot_bytes": (SZ, [CFG, I]),
     "stepq_intb_quantize_pool": (I, [CFG, I, I, P, P, I, P, I, P]),
     "stepq_intb_dequantize_pool": (I, [CFG, I, I, P, I, P, I, P, P]),

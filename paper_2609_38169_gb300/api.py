@@ -230,6 +230,20 @@ def stepq_fp32_decode_step(cfg: Config, layer: int, pool, slots, q, k, v, beta, 
                                             _stream(stream)), "stepq_fp32_decode_step")
 
 
+def stepq_fp32_exact_read_step(cfg: Config, layer: int, pool, read_pool, slots, q, k, v, beta, gate,
+                               y, pool_slots=None, stream=None):
+    import torch
+    f = torch.float32
+    c = cfg.c()
+    ps = pool_slots if pool_slots is not None else pool.shape[0]
+    check(_lib.lib().stepq_fp32_exact_read_step(C.byref(c), layer, _dev_ptr(pool, f),
+                                                _dev_ptr(read_pool, f), int(ps),
+                                                _dev_ptr(slots, torch.int32), slots.numel(),
+                                                _dev_ptr(q, f), _dev_ptr(k, f), _dev_ptr(v, f),
+                                                _dev_ptr(beta, f), _dev_ptr(gate, f), _dev_ptr(y, f),
+                                                _stream(stream)), "stepq_fp32_exact_read_step")
+
+
 def stepq_prefill_fp32(cfg: Config, states, q, k, v, beta, gate, y, stream=None):
     """Chunked prefill over T tokens on FP32 states [B][Hv][128][128] (in place);
     q, k [B][T][Hk][128], v [B][T][Hv][128], beta [B][T][Hv], gate [B][T][Hv]

@@ -95,8 +95,26 @@ extern "C" stepq_status stepq_fp32_decode_step(const stepq_config *cfg, int laye
     if (!aligned(pool, 16)) return STEPQ_ERR_ALIGN;
     if ((st = check_inputs(cfg, q, k, v, beta, gate, y)) != STEPQ_OK) return st;
     if (B == 0) return STEPQ_OK;
-    return launch_fp32_decode(cfg, layer, pool, pool_slots, slots, B, q, k, v, beta, gate, y,
-                              (cudaStream_t)stream);
+    return launch_fp32_decode(cfg, layer, pool, nullptr, pool_slots, slots, B, q, k, v, beta, gate,
+                              y, (cudaStream_t)stream);
+}
+
+extern "C" stepq_status stepq_fp32_exact_read_step(const stepq_config *cfg, int layer, float *pool,
+                                                   const float *read_pool, int pool_slots,
+                                                   const int32_t *slots, int B, const float *q,
+                                                   const float *k, const float *v, const float *beta,
+                                                   const float *gate, float *y,
+                                                   stepq_stream_t stream) {
+    stepq_status st = validate_config(cfg, false);
+    if (st != STEPQ_OK) return st;
+    if (!pool || !read_pool || (B > 0 && !slots) || B < 0 || pool_slots <= 0 || layer < 0 ||
+        layer >= cfg->n_layers || !v || !y)
+        return STEPQ_ERR_ARG;
+    if (!aligned(pool, 16) || !aligned(read_pool, 16)) return STEPQ_ERR_ALIGN;
+    if ((st = check_inputs(cfg, q, k, v, beta, gate, y)) != STEPQ_OK) return st;
+    if (B == 0) return STEPQ_OK;
+    return launch_fp32_decode(cfg, layer, pool, read_pool, pool_slots, slots, B, q, k, v, beta, gate,
+                              y, (cudaStream_t)stream);
 }
 
 extern "C" stepq_status stepq_prefill_fp32(const stepq_config *cfg, int B, int T, float *states,
@@ -113,7 +131,7 @@ extern "C" stepq_status stepq_prefill_fp32(const stepq_config *cfg, int B, int T
 }
 
 extern "C" size_t stepq_intb_slot_bytes(const stepq_config *cfg, int bits) {
-    if (validate_config(cfg, false) != STEPQ_OK || (bits != 4 && bits != 8)) return 0;
+    if (validate_config(cfg, false) != STEPQ_OK || (bits != 4 && bits != 6 && bits != 8)) return 0;
     size_t page = intb_head_bytes(bits) * cfg->n_value_heads * cfg->n_layers;
     return (page + 255) / 256 * 256;
 }
@@ -122,7 +140,7 @@ static stepq_status check_intb(const stepq_config *cfg, int bits, int layer, boo
                                const void *pool, int pool_slots, const int32_t *slots, int B) {
     stepq_status st = validate_config(cfg, false);
     if (st != STEPQ_OK) return st;
-    if (bits != 4 && bits != 8) return STEPQ_ERR_UNSUPPORTED;
+    if (bits != 4 && bits != 6 && bits != 8) return STEPQ_ERR_UNSUPPORTED;
     if (!pool || (B > 0 && !slots) || B < 0 || pool_slots <= 0) return STEPQ_ERR_ARG;
     if (layer < (allow_all ? -1 : 0) || layer >= cfg->n_layers) return STEPQ_ERR_ARG;
     if (!aligned(pool, 256)) return STEPQ_ERR_ALIGN;

@@ -27,6 +27,7 @@ constexpr int kStage = kPage + kVecBytes;
 
 struct DecodeArgs {
     uint8_t *pool;
+    const uint8_t *read_pool;   // exact-read variant: the states the retrieval reads
     uint64_t slot_bytes, layer_off;
     int pool_slots;
     const int32_t *slots;
@@ -42,6 +43,9 @@ __device__ __forceinline__ void row_dup(const float4 *v, int i, uint64_t &xx, ui
     zz = u2pair(q.z, q.w);
 }
 
+// READ: the retrieval reads u = k^T D S_ref from read_pool (same layout)
+// instead of the page's own state; the update still writes D S + beta k (v - u)^T.
+template <bool READ>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     uint64_t *bars = (uint64_t *)(smem + kOffBars);
@@ -73,7 +77,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeArgs a) {
             bulk_load(vec + 256, a.v + ((size_t)b * a.Hv + h) * 128, 512, &bars[s]);
             if (a.gate_per_row) bulk_load(vec + 384, a.gate + ((size_t)b * a.Hv + h) * 128, 512, &bars[s]);
         },
-        [&](int h, int b, int, int s, bool ok, const auto &refill) {
+        [&](int h, int b, int slot, int s, bool ok, const auto &refill) {
             const size_t u = (size_t)b * a.Hv + h;
             const float beta = a.beta[u], gs = a.gate_per_row ? 0.f : a.gate[u];
             float *S = (float *)(stages + (size_t)s * kStage);
@@ -96,8 +100,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeArgs a) {
                 x2[r][0] = fmul2(u2pair(sv.x, sv.y), dd);
                 x2[r][1] = fmul2(u2pair(sv.z, sv.w), dd);
                 uint64_t(&acc)[2] = (r & 1) ? ub : ua;
-                acc[0] = ffma2(kk, x2[r][0], acc[0]);
-                acc[1] = ffma2(kk, x2[r][1], acc[1]);
+                if (READ) {
+                    const float *Sr = (const float *)(a.read_pool + (page_of(h, slot) - a.pool));
+                    const float4 rv = *(const float4 *)&Sr[(16 * w + r) * 128 + 4 * l];
+                    acc[0] = ffma2(kk, fmul2(f2(rv.x, rv.y), dd), acc[0]);
+                    acc[1] = ffma2(kk, fmul2(f2(rv.z, rv.w), dd), acc[1]);
+                } else {
+                    acc[0] = ffma2(kk, x2[r][0], acc[0]);
+                    acc[1] = ffma2(kk, x2[r][1], acc[1]);
+                }
             }
             {
                 const uint64_t s0 = fadd2(ua[0], ub[0]), s1 = fadd2(ua[1], ub[1]);
@@ -145,11 +156,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeArgs a) {
 
 }  // namespace fk
 
-stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool, int pool_slots,
-                                const int32_t *slots, int B, const float *q, const float *k,
-                                const float *v, const float *beta, const float *gate, float *y,
-                                cudaStream_t s) {
+stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool,
+                                const float *read_pool, int pool_slots, const int32_t *slots, int B,
+                                const float *q, const float *k, const float *v, const float *beta,
+                                const float *gate, float *y, cudaStream_t s) {
     fk::DecodeArgs a{};
+    a.read_pool = (const uint8_t *)read_pool;
     const uint64_t per_layer = (uint64_t)fk::kPage * (uint64_t)cfg->n_value_heads;
     a.pool = (uint8_t *)pool;
     a.slot_bytes = per_layer * (uint64_t)cfg->n_layers;
@@ -171,12 +183,13 @@ stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool,
     stages = stages < 2 ? 2 : (stages > 3 ? 3 : stages);
     a.n_stages = stages;
     const int smem = fk::kOffStages + stages * fk::kStage;
-    if (cudaFuncSetAttribute((const void *)fk::decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem) != cudaSuccess)
+    const void *fn = read_pool ? (const void *)fk::decode_kernel<true> : (const void *)fk::decode_kernel<false>;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
         return STEPQ_ERR_CUDA;
     int grid = sms > 0 ? sms : 1;
     if (grid > a.items) grid = a.items;
-    fk::decode_kernel<<<grid, kThreads, smem, s>>>(a);
+    if (read_pool) fk::decode_kernel<true><<<grid, kThreads, smem, s>>>(a);
+    else fk::decode_kernel<false><<<grid, kThreads, smem, s>>>(a);
     return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;
 }
 

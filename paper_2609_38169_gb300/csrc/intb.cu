@@ -4,7 +4,8 @@
 // kernel, so that the comparison measures the codecs and not the plumbing.
 //
 // Tile mapping: warp w owns key rows 16w..16w+15, lane l the value columns
-// 4l..4l+3; a lane's 4 codes of a row are one word (8-bit) or half-word (4-bit).
+// 4l..4l+3; a lane's 4 codes of a row are one word (8-bit), three bytes at
+// byte 3l (6-bit) or a half-word (4-bit).
 // Per row the tile holds Z = q with X_ij = a_i Z_ij, a_i = s_i d_i (d_i the
 // gate), so the decode is the code itself. Every column reduction needs one
 // cross-warp step; the row absmax is a warp reduce-scatter.
@@ -122,6 +123,16 @@ __device__ __forceinline__ void decode_row(const uint8_t *row, int l, uint64_t &
         f1 = __byte_perm(w, kMagicBits, 0x7651);
         f2 = __byte_perm(w, kMagicBits, 0x7652);
         f3 = __byte_perm(w, kMagicBits, 0x7653);
+    } else if (B == 6) {
+        // 24 bits at bit 24 l: a funnel shift of the two words that hold them
+        // (the last lane's upper word is clamped into the row; it is unused).
+        const uint32_t *wd = (const uint32_t *)row;
+        const int wi = (3 * l) >> 2;
+        const uint32_t x = __funnelshift_r(wd[wi], wd[min(wi + 1, 23)], 8 * ((3 * l) & 3));
+        f0 = and_or(x, 0x3Fu, kMagicBits);
+        f1 = and_or(x >> 6, 0x3Fu, kMagicBits);
+        f2 = and_or(x >> 12, 0x3Fu, kMagicBits);
+        f3 = and_or(x >> 18, 0x3Fu, kMagicBits);
     } else {
         const uint32_t x = ((const uint16_t *)row)[l];
         f0 = and_or(x, 0xFu, kMagicBits);
@@ -140,6 +151,14 @@ __device__ __forceinline__ void store_row(uint8_t *row, int l, uint32_t f0, uint
     if (B == 8) {
         const uint32_t lo = __byte_perm(f0, f1, 0x0040), hi = __byte_perm(f2, f3, 0x0040);
         ((uint32_t *)row)[l] = __byte_perm(lo, hi, 0x5410);
+    } else if (B == 6) {
+        // Lane l holds bits 24l..24l+23 of the row; lane t < 24 assembles word t
+        // from lanes floor(4t/3) and the next (offset 0, 8 or 16 bits).
+        constexpr uint32_t K = kMagicBits + (kMagicBits << 6) + (kMagicBits << 12) + (kMagicBits << 18);
+        const uint32_t v = (f0 + (f1 << 6) + (f2 << 12) + (f3 << 18) - K) & 0xFFFFFFu;
+        const int lt = min(l, 23), l0 = (4 * lt) / 3, off = 32 * lt - 24 * l0;
+        const uint32_t a = __shfl_sync(0xffffffffu, v, l0), b = __shfl_sync(0xffffffffu, v, l0 + 1);
+        if (l < 24) ((uint32_t *)row)[l] = (a >> off) | (b << (24 - off));
     } else {
         constexpr uint32_t K = kMagicBits + (kMagicBits << 4) + (kMagicBits << 8) + (kMagicBits << 12);
         ((uint16_t *)row)[l] = (uint16_t)(f0 + (f1 << 4) + (f2 << 8) + (f3 << 12) - K);
@@ -290,6 +309,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a, int b
             const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
             float *y_out = a.y + u * 128;
             if (bits == 8) return decode_item<8>(t, S, st, gs, a.gate_per_row, beta, y_out, ok, refill);
+            if (bits == 6) return decode_item<6>(t, S, st, gs, a.gate_per_row, beta, y_out, ok, refill);
             return decode_item<4>(t, S, st, gs, a.gate_per_row, beta, y_out, ok, refill);
         },
         [&](int h, int slot, int s) {
@@ -303,7 +323,7 @@ stepq_status launch_intb_decode(const stepq_config *cfg, int bits, int layer, ui
                                 int pool_slots, const int32_t *slots, int B, const float *q,
                                 const float *k, const float *v, const float *beta,
                                 const float *gate, float *y, cudaStream_t s) {
-    if (bits != 4 && bits != 8) return STEPQ_ERR_ARG;
+    if (bits != 4 && bits != 6 && bits != 8) return STEPQ_ERR_ARG;
     ib::DecodeArgs a{};
     const uint64_t hb = intb_head_bytes(bits);
     const uint64_t per_layer = hb * (uint64_t)cfg->n_value_heads;

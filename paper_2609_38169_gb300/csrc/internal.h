@@ -110,10 +110,10 @@ stepq_status launch_dequantize_heads(const stepq_plan *p, int layer, const uint8
                                      int pool_slots, const int32_t *slots, int B, float *states,
                                      size_t stride_b, cudaStream_t s);
 // baselines.cu
-stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool, int pool_slots,
-                                const int32_t *slots, int B, const float *q, const float *k,
-                                const float *v, const float *beta, const float *gate, float *y,
-                                cudaStream_t s);
+stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool,
+                                const float *read_pool, int pool_slots, const int32_t *slots, int B,
+                                const float *q, const float *k, const float *v, const float *beta,
+                                const float *gate, float *y, cudaStream_t s);
 stepq_status launch_intb_quantize(const stepq_config *cfg, int bits, int layer,
                                   const float *states, size_t state_stride_b,
                                   const int32_t *slots, int B, uint8_t *pool, int pool_slots,

@@ -31,6 +31,7 @@ VARIANTS = {
     "stepq6": dict(kind="stepq", nominal_bits=6, candidates=(4, 6, 8)),
     "stepq4": dict(kind="stepq", nominal_bits=4, candidates=(2, 4, 6, 8)),
     "int8": dict(kind="intb", bits=8),
+    "int6": dict(kind="intb", bits=6),
     "int4": dict(kind="intb", bits=4),
 }
 # Component ablations of Sec. 5.4 that the plan alone expresses: the spatial

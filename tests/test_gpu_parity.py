@@ -117,7 +117,39 @@ def test_fp32_state_decode(torch):
     assert np.abs(got - S_o).max() <= 1e-5 * np.abs(S_o).max()
 
 
-@pytest.mark.parametrize("bits,name", [(8, "gqa"), (4, "channel")])
+@pytest.mark.parametrize("name", ["gqa", "channel"])
+def test_fp32_exact_read_decode(torch, name):
+    """Exact-read step of the feedback experiment (App. B.4): the residual reads
+    a separate reference pool, which the kernel leaves untouched."""
+    wl = W.WORKLOADS[name]
+    cfg = A.Config.from_workload(wl)
+    mp = W.model_params(wl)
+    B = 12
+    slots = _slots(wl, B)
+    S_ref = W.random_states(wl, B * wl.hv).reshape(B, wl.hv, 128, 128)
+    rng = np.random.default_rng(11)
+    S = (S_ref + 0.05 * np.abs(S_ref).max() * rng.standard_normal(S_ref.shape)).astype(np.float32)
+    pool = np.zeros((wl.pool_slots, 1, wl.hv, 128, 128), np.float32)
+    rpool = np.zeros_like(pool)
+    pool[slots, 0] = S
+    rpool[slots, 0] = S_ref
+    (pool_d, rpool_d, slots_d) = to_dev(pool, rpool, slots)
+    inp = W.step_inputs(wl, mp, W.STREAM_DECODE, 3, 0, batch=B)
+    q, k, v, beta, gate = to_dev(inp.q, inp.k, inp.v, inp.beta, inp.gate)
+    y_d = torch.empty((B, wl.hv, 128), dtype=torch.float32, device="cuda")
+    A.stepq_fp32_exact_read_step(cfg, 0, pool_d, rpool_d, slots_d, q, k, v, beta, gate, y_d)
+    S_o = S.copy()
+    y_o = O.delta_batch_read(S_o, S_ref, inp.q, inp.k, inp.v, inp.beta, inp.gate)
+    t = Tally()
+    compare_y(t, y_d.cpu().numpy(), y_o)
+    assert t.y_worst <= 1e-5
+    got = pool_d.cpu().numpy()[slots, 0]
+    assert np.abs(got - S_o).max() <= 1e-5 * np.abs(S_o).max()
+    assert np.array_equal(rpool_d.cpu().numpy(), rpool)
+    assert A.stepq_device_error() == 0
+
+
+@pytest.mark.parametrize("bits,name", [(8, "gqa"), (4, "channel"), (6, "gqa"), (6, "channel")])
 def test_intb_decode(torch, bits, name):
     """Uniform rowwise-absmax INT-b state (App. B.5), teacher-forced for 3 steps."""
     wl = W.WORKLOADS[name]

@@ -96,8 +96,12 @@ def test_argument_errors_before_launch():
     assert L.stepq_decode_step(None, 0, None, 1, None, 1, None, None, None, None, None, None, None) == 1
     assert L.stepq_fp32_decode_step(C.byref(cfg), 5, C.c_void_p(256), 1, C.c_void_p(256), 1,
                                     None, None, None, None, None, None, None) == 1
+    assert L.stepq_fp32_exact_read_step(C.byref(cfg), 0, C.c_void_p(256), None, 1, C.c_void_p(256), 1,
+                                        None, None, C.c_void_p(256), None, None, C.c_void_p(256),
+                                        None) == 1
     assert L.stepq_intb_slot_bytes(C.byref(cfg), 3) == 0
     assert L.stepq_intb_slot_bytes(C.byref(cfg), 8) == (256 + 128 * 128) * 4
+    assert L.stepq_intb_slot_bytes(C.byref(cfg), 6) == (256 + 128 * 96) * 4
     assert L.stepq_status_str(2) == b"slot id out of range"
 
 
@@ -118,11 +122,22 @@ def test_host_only_plan_refuses_device_calls(oracle):
 def test_drift_variants_and_cli():
     """The drift module's variant table and command line (no device work)."""
     from paper_2609_38169_gb300 import drift
-    assert set(drift.VARIANTS) == {"stepq6", "stepq4", "int8", "int4"}
+    assert set(drift.VARIANTS) == {"stepq6", "stepq4", "int8", "int6", "int4"}
     assert drift.VARIANTS["stepq4"]["candidates"] == (2, 4, 6, 8)
     with pytest.raises(SystemExit) as e:
         drift.main(["--help"])
     assert e.value.code == 0
+
+
+def test_feedback_cli():
+    """The feedback-experiment module's command line (no device work)."""
+    from paper_2609_38169_gb300 import feedback
+    with pytest.raises(SystemExit) as e:
+        feedback.main(["--help"])
+    assert e.value.code == 0
+    with pytest.raises(SystemExit) as e:
+        feedback.main(["--codecs", "int5"])
+    assert e.value.code == 2
 
 
 def test_measure_cli():

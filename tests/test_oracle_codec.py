@@ -219,7 +219,7 @@ def test_column_update_minimises_weighted_error(oracle, rng, unit):
         assert abs(0.5 * (lo + hi) - c[j]) <= 1e-5 * c[j]
 
 
-@pytest.mark.parametrize("bits", [4, 8])
+@pytest.mark.parametrize("bits", [4, 6, 8])
 def test_intb_baseline(oracle, rng, bits):
     """App. B.5: per key row s_i = fp16(absmax/q_b) in [2^-14, 65504], nearest codes."""
     X = _state(rng)

@@ -72,6 +72,52 @@ def test_directional_contraction(oracle, rng):
 
 
 @pytest.mark.parametrize("per_row", [False, True])
+def test_exact_read_error_is_only_decayed(oracle, rng, per_row):
+    """App. B.4: with the residual reading the reference state, the path's error
+    evolves as E_t = D_t E_{t-1}, while the native step gives (I - beta k k^T) D E."""
+    S_ref = (rng.standard_normal((D, D)) * np.exp(rng.normal(size=(D, 1)))).astype(np.float32)
+    E = (1e-2 * rng.standard_normal((D, D)) * np.abs(S_ref).max()).astype(np.float32)
+    S = (S_ref.astype(np.float64) + E).astype(np.float32)
+    E = S.astype(np.float64) - S_ref.astype(np.float64)
+    q, k, v, beta, gate = _inputs(rng, per_row)
+    # reference trajectory: the plain step of S_ref, written out here in fp64
+    g = np.broadcast_to(gate.astype(np.float64), (D,))
+    k64, b = k.astype(np.float64), float(beta)
+    P_ref = g[:, None] * S_ref.astype(np.float64)
+    ref1 = P_ref + b * np.outer(k64, v.astype(np.float64) - k64 @ P_ref)
+    S1, y = oracle.delta_step_read(S, S_ref, q, k, v, beta, gate)
+    scale = np.abs(ref1).max()
+    assert np.abs((S1 - ref1) - g[:, None] * E).max() <= 1e-6 * scale
+    assert np.abs(y - S1.astype(np.float64).T @ q.astype(np.float64)).max() <= 1e-6 * np.abs(y).max()
+    # the native step of the same perturbed state removes the k-direction of D E
+    N1, _ = oracle.delta_step(S, q, k, v, beta, gate)
+    DE = g[:, None] * E
+    assert np.abs((N1 - ref1) - (DE - b * np.outer(k64, k64 @ DE))).max() <= 1e-6 * scale
+    # and with S = S_ref the two steps coincide
+    X1, _ = oracle.delta_step_read(S_ref, S_ref, q, k, v, beta, gate)
+    R1, _ = oracle.delta_step(S_ref, q, k, v, beta, gate)
+    assert np.abs(X1 - R1).max() <= 4e-7 * scale
+
+
+def test_exact_read_batch_matches_single_steps(oracle, rng):
+    n, Hk, Hv = 2, 1, 2
+    S = rng.standard_normal((n, Hv, D, D)).astype(np.float32)
+    S_ref = (S + 0.1 * rng.standard_normal(S.shape)).astype(np.float32)
+    q = rng.standard_normal((n, Hk, D)).astype(np.float32)
+    k = rng.standard_normal((n, Hk, D)).astype(np.float32) / np.sqrt(D)
+    v = rng.standard_normal((n, Hv, D)).astype(np.float32)
+    beta = rng.uniform(0.1, 0.9, (n, Hv)).astype(np.float32)
+    gate = rng.uniform(0.8, 1.0, (n, Hv, D)).astype(np.float32)
+    Sb = S.copy()
+    y = oracle.delta_batch_read(Sb, S_ref, q, k, v, beta, gate)
+    for b in range(n):
+        for h in range(Hv):
+            s1, y1 = oracle.delta_step_read(S[b, h], S_ref[b, h], q[b, 0], k[b, 0], v[b, h],
+                                            beta[b, h], gate[b, h])
+            assert np.array_equal(Sb[b, h], s1) and np.array_equal(y[b, h], y1)
+
+
+@pytest.mark.parametrize("per_row", [False, True])
 def test_row_impact_closed_form_and_readout_identity(oracle, rng, per_row):
     """g_t = A_t^T q_t (Sec. 4.1; Eq. kda_sensitivity) and the App. B.3 identity:
     a unit-norm perturbation confined to key row i changes the next readout by
