@@ -1,5 +1,5 @@
 """Measurements of the kernels beside the headline decode step (which bench.py
-times): the row-unit decode step against the FP32-state and INT8 comparison
+times): the row-unit decode step against the FP32-state and INT-b comparison
 kernels on one layer of a channel-gate pool, and the chunked FP32 prefill.
 Each subcommand prints one JSON line; inputs are synthetic (the workload
 generators), resident on the device, and timed with CUDA events after warm-up.
@@ -35,7 +35,7 @@ def _timeit(fn, n=20, warmup=3):
 def rows(slots=1024, bits=6):
     """One layer of the drift workload's shape (32 heads, channel gates) over
     `slots` slots in a random permutation: STEPQuant row units against the
-    FP32-state and INT8 rowwise kernels on identical inputs."""
+    FP32-state and INT8 / INT6 rowwise kernels on identical inputs."""
     import torch
     dev = torch.device("cuda")
     wl = W.WORKLOADS["drift"].replace(layers=1, batch=slots, pool_slots=slots, nominal_bits=bits,
@@ -67,12 +67,14 @@ def rows(slots=1024, bits=6):
     t = _timeit(lambda: A.stepq_fp32_decode_step(cfg, 0, ref, perm, q, k, v, beta, gate, y))
     out["kernels"]["fp32_state"] = {"us_per_launch": t * 1e6, "value": units / t,
                                     "algorithmic_gbs": units * (2 * 4 * D * D + vec) / t / 1e9}
-    sb = A.stepq_intb_slot_bytes(cfg, 8)
-    pi = torch.zeros(slots * sb, dtype=torch.uint8, device=dev)
-    A.stepq_intb_quantize_pool(cfg, 8, -1, S, all_slots, pi)
-    t = _timeit(lambda: A.stepq_intb_decode_step(cfg, 8, 0, pi, perm, q, k, v, beta, gate, y))
-    out["kernels"]["int8_rowwise"] = {"us_per_launch": t * 1e6, "value": units / t,
-                                      "algorithmic_gbs": units * (2 * sb / wl.hv + vec) / t / 1e9}
+    for b in (8, 6):
+        sb = A.stepq_intb_slot_bytes(cfg, b)
+        pi = torch.zeros(slots * sb, dtype=torch.uint8, device=dev)
+        A.stepq_intb_quantize_pool(cfg, b, -1, S, all_slots, pi)
+        t = _timeit(lambda: A.stepq_intb_decode_step(cfg, b, 0, pi, perm, q, k, v, beta, gate, y))
+        out["kernels"][f"int{b}_rowwise"] = {"us_per_launch": t * 1e6, "value": units / t,
+                                             "algorithmic_gbs": units * (2 * sb / wl.hv + vec) / t / 1e9}
+        del pi
     assert A.stepq_device_error() == 0
     return out
 
