@@ -84,6 +84,9 @@ def _declare(L):
         "or_intb_encode_head": (None, [P, I, P]),
         "or_intb_decode_head": (None, [P, I, P]),
         "or_intb_step_head": (None, [P, I, P, P, P, F, P, I, P]),
+        "or_temporal_head_bytes": (C.c_size_t, [P]),
+        "or_temporal_encode_head": (None, [P, P, P]),
+        "or_temporal_decode_head": (None, [P, P, P]),
         "or_row_weights": (None, [I, P, P]),
         "or_lifetime_weight": (D_, [D_, I]),
         "or_allocate_dp": (I, [I, I, P, LL, P, P]),
@@ -290,6 +293,25 @@ def intb_step_head(page, bits, q, k, v, beta, gate):
 
 
 # --------------------------------------------------------------------- plan
+def temporal_head_bytes(rb) -> int:
+    return lib().or_temporal_head_bytes(_p(_i8(rb)))
+
+
+def temporal_encode_head(X, rb) -> np.ndarray:
+    """"Temporal only" ablation codec (Sec. 5.4): the plan's row widths rb (16 =
+    FP16 pivot) with the rowwise absmax quantizer of App. B.5."""
+    rb = _i8(rb)
+    page = np.zeros(temporal_head_bytes(rb), np.uint8)
+    lib().or_temporal_encode_head(_p(_f32(X)), _p(rb), _p(page))
+    return page
+
+
+def temporal_decode_head(page, rb) -> np.ndarray:
+    S = np.zeros((D, D), np.float64)
+    lib().or_temporal_decode_head(_p(np.ascontiguousarray(page, np.uint8)), _p(_i8(rb)), _p(S))
+    return S
+
+
 def row_weights(omega) -> np.ndarray:
     om = _f32(omega)
     w = np.zeros_like(om)

@@ -392,3 +392,62 @@ void or_intb_step_head(uint8_t *page, int bits, const float *q, const float *k, 
     free(S);
     free(X);
 }
+
+/* ---- "Temporal only" ablation codec (Sec. 5.4) ----
+ * The plan's calibrated widths and FP16 pivots, with the uniform baseline's
+ * rowwise quantizer (App. B.5) in place of the dual-axis fit: a key row of
+ * width b < 16 stores s_i = fp16(clamp(absmax_i / q_b)) and nearest codes of
+ * X * fp32(1/s_i) in [-q_b, q_b]; a pivot row (b = 16) stores fp16(X) and s_i = 0.
+ * Head segment: s[128] fp16 | row i in index order, 16 b_i bytes (offset-binary
+ * codes LSB-first, or 128 fp16 values). rb: the 128 row widths. */
+size_t or_temporal_head_bytes(const int8_t *rb)
+{
+    size_t n = 256;
+    for (int i = 0; i < OR_D; i++)
+        n += (size_t)16 * rb[i];
+    return n;
+}
+
+void or_temporal_encode_head(const float *X, const int8_t *rb, uint8_t *page)
+{
+    uint8_t *row = page + 256;
+    for (int i = 0; i < OR_D; i++) {
+        int b = rb[i];
+        if (b == OR_PIVOT_BITS) {
+            put_u16(page + 2 * i, 0);
+            for (int j = 0; j < OR_D; j++)
+                put_u16(row + 2 * j, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
+        } else {
+            int qm = qmax_of(b);
+            float amax = 0.0f;
+            for (int j = 0; j < OR_D; j++)
+                if (fabsf(X[i * OR_D + j]) > amax)
+                    amax = fabsf(X[i * OR_D + j]);
+            double s16 = or_fp16_round(clampd((float)((double)amax / qm), F16_MIN_NORMAL, F16_MAX));
+            float inv = (float)(1.0 / s16);
+            put_u16(page + 2 * i, or_fp16_encode(s16));
+            for (int j = 0; j < OR_D; j++) {
+                int qv = (int)clampd(rint((double)mul32(X[i * OR_D + j], inv)), -qm, qm);
+                put_bits(row, j * b, b, (unsigned)(qv + (1 << (b - 1))));
+            }
+        }
+        row += (size_t)16 * b;
+    }
+}
+
+void or_temporal_decode_head(const uint8_t *page, const int8_t *rb, double *S)
+{
+    const uint8_t *row = page + 256;
+    for (int i = 0; i < OR_D; i++) {
+        int b = rb[i];
+        if (b == OR_PIVOT_BITS) {
+            for (int j = 0; j < OR_D; j++)
+                S[i * OR_D + j] = or_fp16_decode(get_u16(row + 2 * j));
+        } else {
+            double s = or_fp16_decode(get_u16(page + 2 * i));
+            for (int j = 0; j < OR_D; j++)
+                S[i * OR_D + j] = s * (double)((int)get_bits(row, j * b, b) - (1 << (b - 1)));
+        }
+        row += (size_t)16 * b;
+    }
+}

@@ -80,6 +80,9 @@ void or_unpack_head(const uint8_t *page, int unit_kind, const int8_t *row_bits,
 size_t or_intb_head_bytes(int bits);
 void or_intb_encode_head(const float *X, int bits, uint8_t *page);
 void or_intb_decode_head(const uint8_t *page, int bits, double *S);
+size_t or_temporal_head_bytes(const int8_t *rb);
+void or_temporal_encode_head(const float *X, const int8_t *rb, uint8_t *page);
+void or_temporal_decode_head(const uint8_t *page, const int8_t *rb, double *S);
 void or_intb_step_head(uint8_t *page, int bits, const float *q, const float *k, const float *v,
                        float beta, const float *gate, int gate_per_row, float *y);
 

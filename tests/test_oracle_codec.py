@@ -235,3 +235,47 @@ def test_intb_baseline(oracle, rng, bits):
     arg = np.abs(X).argmax(axis=1)
     assert np.all(np.abs(q[np.arange(D), arg]) == qm)
     assert np.all(np.abs(R - X) <= s[:, None] * (0.5 + 1e-5) + (np.abs(q) == qm) * np.abs(X))
+
+
+@pytest.mark.parametrize("bits", [4, 6, 8])
+def test_temporal_uniform_widths_is_intb(oracle, rng, bits):
+    """"Temporal only" (Sec. 5.4) at one width without pivots is the uniform
+    rowwise baseline of App. B.5, byte for byte."""
+    X = _state(rng)
+    rb = np.full(D, bits, np.int8)
+    page = oracle.temporal_encode_head(X, rb)
+    assert np.array_equal(page, oracle.intb_encode_head(X, bits))
+    assert np.array_equal(oracle.temporal_decode_head(page, rb), oracle.intb_decode_head(page, bits))
+
+
+def test_temporal_mixed_widths_and_pivots(oracle, rng):
+    """Mixed row widths with FP16 pivot rows: every row follows App. B.5 at its
+    own width (numpy scale, absmax at +-q_b, half-step bound), pivots are numpy
+    float16, and rows sit in index order (independent numpy unpacker)."""
+    X = _state(rng)
+    rb = rng.choice([2, 4, 6, 8, PIV], size=D, p=[0.15, 0.3, 0.3, 0.2, 0.05]).astype(np.int8)
+    rb[:2] = (PIV, 2)
+    page = oracle.temporal_encode_head(X, rb)
+    assert page.size == 256 + 16 * int(rb.astype(np.int64).sum())
+    R = oracle.temporal_decode_head(page, rb)
+    s = page[:256].view(np.float16).astype(np.float64)
+    bits = np.unpackbits(page, bitorder="little")
+    off = 256
+    for i in range(D):
+        b = int(rb[i])
+        x = X[i].astype(np.float64)
+        if b == PIV:
+            assert s[i] == 0
+            vals = page[off:off + 256].view(np.float16).astype(np.float64)
+            assert np.array_equal(vals, np.float16(X[i]).astype(np.float64))
+            assert np.array_equal(R[i], vals)
+        else:
+            qm = 2 ** (b - 1) - 1
+            assert s[i] == np.float16(np.clip(np.abs(x).max() / qm, 2 ** -14, 65504))
+            u = bits[8 * off:8 * off + b * D].reshape(D, b) @ (1 << np.arange(b))
+            q = u.astype(np.int64) - (1 << (b - 1))
+            assert np.all(np.abs(q) <= qm) and abs(q[np.abs(x).argmax()]) == qm
+            assert np.array_equal(R[i], s[i] * q)
+            assert np.all(np.abs(R[i] - x) <= s[i] * (0.5 + 1e-5) + (np.abs(q) == qm) * np.abs(x))
+        off += 16 * b
+    assert off == page.size
