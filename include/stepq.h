@@ -209,6 +209,25 @@ stepq_status stepq_fp32_exact_read_step(const stepq_config *cfg, int layer, floa
                                         const float *k, const float *v, const float *beta,
                                         const float *gate, float *y, stepq_stream_t stream);
 
+/* "Temporal only" ablation state (Sec. 5.4): the plan's calibrated widths
+ * and FP16 pivots, with the uniform rowwise quantizer of App. B.5 in place of
+ * the dual-axis fit. A key row of width b < 16 stores s_i = fp16(clamp(
+ * absmax_i / q_b, 2^-14, 65504)) and nearest codes of X * fp32(1/s_i) in
+ * [-q_b, q_b] (offset-binary, LSB-first); a pivot row stores fp16(X) with
+ * s_i = 0. Head segment: s[128] fp16 | row i in index order, 16 b_i bytes;
+ * segments in (layer, head) order; slot stride = stepq_temporal_slot_bytes()
+ * (a multiple of 256; 0 for a null plan). States, slots, layer = -1 and the
+ * errors behave as in stepq_quantize_pool / stepq_dequantize_pool. A decode
+ * step with this codec is dequantize, stepq_fp32_decode_step, quantize: it
+ * serves accuracy ablations and has no fused kernel. */
+size_t stepq_temporal_slot_bytes(const stepq_plan *plan);
+stepq_status stepq_temporal_quantize_pool(const stepq_plan *plan, int layer, const float *states,
+                                          const int32_t *slots, int B, void *pool, int pool_slots,
+                                          stepq_stream_t stream);
+stepq_status stepq_temporal_dequantize_pool(const stepq_plan *plan, int layer, const void *pool,
+                                            int pool_slots, const int32_t *slots, int B,
+                                            float *states_out, stepq_stream_t stream);
+
 /* Uniform rowwise-absmax INT-b state (App. B.5): per key row an FP16 scale
  * absmax/q_b clamped to [2^-14, 65504], nearest codes in [-q_b, q_b]. Head
  * segment: s[128] fp16 | 128 rows x 16b bytes; segments in (layer, head)

@@ -39,6 +39,9 @@ SIGNATURES = {
     "stepq_plan_destroy": (None, [P]),
     "stepq_quantize_pool": (I, [P, I, P, P, I, P, I, P]),
     "stepq_dequantize_pool": (I, [P, I, P, I, P, I, P, P]),
+    "stepq_temporal_slot_bytes": (SZ, [P]),
+    "stepq_temporal_quantize_pool": (I, [P, I, P, P, I, P, I, P]),
+    "stepq_temporal_dequantize_pool": (I, [P, I, P, I, P, I, P, P]),
     "stepq_decode_step": (I, [P, I, P, I, P, I, P, P, P, P, P, P, P]),
     "stepq_fp32_decode_step": (I, [CFG, I, P, I, P, I, P, P, P, P, P, P, P]),
     "stepq_prefill_fp32": (I, [CFG, I, I, P, P, P, P, P, P, P, P]),

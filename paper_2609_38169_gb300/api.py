@@ -204,6 +204,31 @@ def stepq_dequantize_pool(plan: Plan, layer: int, pool, slots, states_out, pool_
           "stepq_dequantize_pool")
 
 
+def stepq_temporal_slot_bytes(plan: Plan) -> int:
+    return int(_lib.lib().stepq_temporal_slot_bytes(plan.handle))
+
+
+def stepq_temporal_quantize_pool(plan: Plan, layer: int, states, slots, pool, pool_slots=None,
+                                 stream=None):
+    import torch
+    stride = stepq_temporal_slot_bytes(plan)
+    check(_lib.lib().stepq_temporal_quantize_pool(plan.handle, layer, _dev_ptr(states, torch.float32),
+                                                  _dev_ptr(slots, torch.int32), slots.numel(),
+                                                  _dev_ptr(pool), _pool_slots(pool, stride, pool_slots),
+                                                  _stream(stream)), "stepq_temporal_quantize_pool")
+
+
+def stepq_temporal_dequantize_pool(plan: Plan, layer: int, pool, slots, states_out, pool_slots=None,
+                                   stream=None):
+    import torch
+    stride = stepq_temporal_slot_bytes(plan)
+    check(_lib.lib().stepq_temporal_dequantize_pool(plan.handle, layer, _dev_ptr(pool),
+                                                    _pool_slots(pool, stride, pool_slots),
+                                                    _dev_ptr(slots, torch.int32), slots.numel(),
+                                                    _dev_ptr(states_out, torch.float32),
+                                                    _stream(stream)), "stepq_temporal_dequantize_pool")
+
+
 def stepq_decode_step(plan: Plan, layer: int, pool, slots, q, k, v, beta, gate, y,
                       pool_slots=None, stream=None):
     import torch

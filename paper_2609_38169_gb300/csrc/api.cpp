@@ -69,6 +69,50 @@ extern "C" stepq_status stepq_dequantize_pool(const stepq_plan *p, int layer, co
     return STEPQ_OK;
 }
 
+extern "C" size_t stepq_temporal_slot_bytes(const stepq_plan *p) { return p ? p->t_slot_stride : 0; }
+
+extern "C" stepq_status stepq_temporal_quantize_pool(const stepq_plan *p, int layer,
+                                                     const float *states, const int32_t *slots,
+                                                     int B, void *pool, int pool_slots,
+                                                     stepq_stream_t stream) {
+    stepq_status st = check_plan_call(p, layer, true, pool, pool_slots, slots, B);
+    if (st != STEPQ_OK) return st;
+    if (!states) return STEPQ_ERR_ARG;
+    if (!aligned(states, 16)) return STEPQ_ERR_ALIGN;
+    if (B == 0) return STEPQ_OK;
+    const size_t per_layer = (size_t)p->cfg.n_value_heads * kN;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (layer >= 0)
+        return launch_temporal_quantize(p, layer, states, per_layer, slots, B, (uint8_t *)pool, pool_slots, s);
+    for (int l = 0; l < p->cfg.n_layers; l++)
+        if ((st = launch_temporal_quantize(p, l, states + l * per_layer, per_layer * p->cfg.n_layers,
+                                           slots, B, (uint8_t *)pool, pool_slots, s)) != STEPQ_OK)
+            return st;
+    return STEPQ_OK;
+}
+
+extern "C" stepq_status stepq_temporal_dequantize_pool(const stepq_plan *p, int layer,
+                                                       const void *pool, int pool_slots,
+                                                       const int32_t *slots, int B, float *states,
+                                                       stepq_stream_t stream) {
+    stepq_status st = check_plan_call(p, layer, true, pool, pool_slots, slots, B);
+    if (st != STEPQ_OK) return st;
+    if (!states) return STEPQ_ERR_ARG;
+    if (!aligned(states, 16)) return STEPQ_ERR_ALIGN;
+    if (B == 0) return STEPQ_OK;
+    const size_t per_layer = (size_t)p->cfg.n_value_heads * kN;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (layer >= 0)
+        return launch_temporal_dequantize(p, layer, (const uint8_t *)pool, pool_slots, slots, B, states,
+                                          per_layer, s);
+    for (int l = 0; l < p->cfg.n_layers; l++)
+        if ((st = launch_temporal_dequantize(p, l, (const uint8_t *)pool, pool_slots, slots, B,
+                                             states + l * per_layer, per_layer * p->cfg.n_layers,
+                                             s)) != STEPQ_OK)
+            return st;
+    return STEPQ_OK;
+}
+
 extern "C" stepq_status stepq_decode_step(const stepq_plan *p, int layer, void *pool,
                                           int pool_slots, const int32_t *slots, int B,
                                           const float *q, const float *k, const float *v,

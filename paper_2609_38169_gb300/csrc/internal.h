@@ -59,6 +59,12 @@ struct stepq_plan {
     uint8_t *d_row_bits = nullptr;
     uint32_t *d_row_off = nullptr;
     uint32_t *d_row_slot = nullptr;
+    // layout of the "Temporal only" ablation codec (rowwise absmax at the plan's
+    // widths): head segments in (layer, head) order, rows in index order
+    std::vector<uint64_t> t_head_off;
+    size_t t_slot_stride = 0;
+    uint64_t *d_t_head_off = nullptr;
+    uint32_t *d_t_row_off = nullptr;   // [heads][128] row payload offset within the head segment
 
     stepq::LayerTables layer(int l) const {
         const size_t Hv = (size_t)cfg.n_value_heads;
@@ -114,6 +120,12 @@ stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool,
                                 const float *read_pool, int pool_slots, const int32_t *slots, int B,
                                 const float *q, const float *k, const float *v, const float *beta,
                                 const float *gate, float *y, cudaStream_t s);
+stepq_status launch_temporal_quantize(const stepq_plan *p, int layer, const float *states,
+                                      size_t state_stride_b, const int32_t *slots, int B,
+                                      uint8_t *pool, int pool_slots, cudaStream_t s);
+stepq_status launch_temporal_dequantize(const stepq_plan *p, int layer, const uint8_t *pool,
+                                        int pool_slots, const int32_t *slots, int B, float *states,
+                                        size_t state_stride_b, cudaStream_t s);
 stepq_status launch_intb_quantize(const stepq_config *cfg, int bits, int layer,
                                   const float *states, size_t state_stride_b,
                                   const int32_t *slots, int B, uint8_t *pool, int pool_slots,

@@ -323,6 +323,21 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
     }
     p->slot_stride = (size_t)((off + 255) / 256 * 256);
 
+    // "Temporal only" layout: s[128] fp16, then row i (index order) in 16 b_i bytes.
+    std::vector<uint32_t> t_row_off(heads * kD);
+    p->t_head_off.resize(heads);
+    uint64_t t_off = 0;
+    for (size_t h = 0; h < heads; h++) {
+        uint32_t bytes = 256;
+        for (int i = 0; i < kD; i++) {
+            t_row_off[h * kD + i] = bytes;
+            bytes += 16u * row_bits[h * kD + i];
+        }
+        p->t_head_off[h] = t_off;
+        t_off += bytes;
+    }
+    p->t_slot_stride = (size_t)((t_off + 255) / 256 * 256);
+
     // Device tables.
     std::vector<float> w2(heads * kD), wis(heads * kD);
     for (size_t t = 0; t < heads * kD; t++) {
@@ -334,7 +349,8 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
     size_t o_w2 = 0, o_wis = align(o_w2 + heads * kD * 4), o_off = align(o_wis + heads * kD * 4),
            o_hb = align(o_off + heads * 8), o_hbits = align(o_hb + heads * 4),
            o_rbits = align(o_hbits + heads), o_roff = align(o_rbits + heads * kD),
-           o_rslot = align(o_roff + heads * kD * 4), total = align(o_rslot + heads * kD * 4);
+           o_rslot = align(o_roff + heads * kD * 4), o_thoff = align(o_rslot + heads * kD * 4),
+           o_troff = align(o_thoff + heads * 8), total = align(o_troff + heads * kD * 4);
     std::vector<uint8_t> host(total, 0);
     std::memcpy(host.data() + o_w2, w2.data(), heads * kD * 4);
     std::memcpy(host.data() + o_wis, wis.data(), heads * kD * 4);
@@ -344,6 +360,8 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
     std::memcpy(host.data() + o_rbits, row_bits.data(), heads * kD);
     std::memcpy(host.data() + o_roff, row_off.data(), heads * kD * 4);
     std::memcpy(host.data() + o_rslot, row_slot.data(), heads * kD * 4);
+    std::memcpy(host.data() + o_thoff, p->t_head_off.data(), heads * 8);
+    std::memcpy(host.data() + o_troff, t_row_off.data(), heads * kD * 4);
     int n_dev = 0;
     if (cudaGetDeviceCount(&n_dev) != cudaSuccess || n_dev == 0) {
         cudaGetLastError();          // host-only plan: its device calls return STEPQ_ERR_CUDA
@@ -366,6 +384,8 @@ extern "C" stepq_status stepq_fit_scales(const stepq_config *cfg, const stepq_ca
     p->d_row_bits = base + o_rbits;
     p->d_row_off = (uint32_t *)(base + o_roff);
     p->d_row_slot = (uint32_t *)(base + o_rslot);
+    p->d_t_head_off = (uint64_t *)(base + o_thoff);
+    p->d_t_row_off = (uint32_t *)(base + o_troff);
     *out = p;
     return STEPQ_OK;
 }

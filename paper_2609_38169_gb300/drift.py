@@ -5,7 +5,8 @@ recurrence (the drift workload: 4 layers x 32 heads with per-key-channel gates,
 Every variant starts from the same FP32 state (warm-up steps from zero on the
 warm-up stream), is quantized once, and then runs free: each step reads its own
 compressed state, updates it and writes it back (STEPQuant: App. C.3 steps 1-7;
-uniform INT-b: the rowwise absmax codec of App. B.5). The FP32-state kernel runs
+uniform INT-b: the rowwise absmax codec of App. B.5; the component ablations of
+Sec. 5.4, listed in ABLATIONS). The FP32-state kernel runs
 beside them on identical inputs. Every `every` steps the relative readout error
 ||y - y_fp32|| / ||y_fp32|| over all layers, slots and heads is recorded, for
 that step and as the RMS over the window since the previous record (the
@@ -34,12 +35,18 @@ VARIANTS = {
     "int6": dict(kind="intb", bits=6),
     "int4": dict(kind="intb", bits=4),
 }
-# Component ablations of Sec. 5.4 that the plan alone expresses: the spatial
-# codec at one uniform width without pivots ("Spatial only"), and the full
-# allocation without its FP16 pivots.
+# Component ablations of Sec. 5.4: "Spatial only" is the dual-axis codec at one
+# uniform width without pivots; "Temporal only" is the calibrated allocation
+# with its FP16 pivots under the rowwise absmax quantizer of App. B.5, and
+# "Temporal w/o pivots" the same without pivots. STEPQuant without its pivots
+# is added beside them.
 ABLATIONS = {
     "spatial6": dict(kind="stepq", nominal_bits=6, candidates=(6,), n_pivots=0),
     "spatial4": dict(kind="stepq", nominal_bits=4, candidates=(4,), n_pivots=0),
+    "temporal6": dict(kind="temporal", nominal_bits=6, candidates=(4, 6, 8)),
+    "temporal4": dict(kind="temporal", nominal_bits=4, candidates=(2, 4, 6, 8)),
+    "temporal6_nopiv": dict(kind="temporal", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0),
+    "temporal4_nopiv": dict(kind="temporal", nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=0),
     "stepq6_nopiv": dict(kind="stepq", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0),
     "stepq4_nopiv": dict(kind="stepq", nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=0),
 }
@@ -52,15 +59,24 @@ class _Variant:
         self.name = name
         self.kind = spec["kind"]
         L = wl.layers
-        if self.kind == "stepq":
+        if self.kind in ("stepq", "temporal"):
             wlv = wl.replace(nominal_bits=spec["nominal_bits"], candidates=spec["candidates"],
                              n_pivots=spec.get("n_pivots", wl.n_pivots))
             self.cfg = A.Config.from_workload(wlv)
             st = A.calibrate(self.cfg, wlv, device, device_inputs=True, **calib)
             self.plan = A.stepq_fit_scales(self.cfg, st.omega, st.mean_log_ret, st.dist, st.pivot)
+        if self.kind == "stepq":
             self.pool = A.alloc_pool(self.plan, slots.numel(), device)
             A.stepq_quantize_pool(self.plan, -1, ref, slots, self.pool)
             self.slot_bytes = self.plan.slot_stride
+        elif self.kind == "temporal":
+            # dequantize, FP32 step, quantize, through a one-layer dense scratch
+            self.slot_bytes = A.stepq_temporal_slot_bytes(self.plan)
+            self.pool = torch.zeros(slots.numel() * self.slot_bytes, dtype=torch.uint8, device=device)
+            A.stepq_temporal_quantize_pool(self.plan, -1, ref, slots, self.pool)
+            self.cfg1 = A.Config.from_workload(wl.replace(layers=1))
+            self.dense = torch.empty((slots.numel(), 1, wl.hv, D, D), dtype=torch.float32, device=device)
+            self.dense_slots = torch.arange(slots.numel(), dtype=torch.int32, device=device)
         else:
             self.bits = spec["bits"]
             self.cfg = A.Config.from_workload(wl)
@@ -72,6 +88,10 @@ class _Variant:
     def step(self, layer, slots, q, k, v, beta, gate, y):
         if self.kind == "stepq":
             A.stepq_decode_step(self.plan, layer, self.pool, slots, q, k, v, beta, gate, y)
+        elif self.kind == "temporal":
+            A.stepq_temporal_dequantize_pool(self.plan, layer, self.pool, slots, self.dense)
+            A.stepq_fp32_decode_step(self.cfg1, 0, self.dense, self.dense_slots, q, k, v, beta, gate, y)
+            A.stepq_temporal_quantize_pool(self.plan, layer, self.dense, slots, self.pool)
         else:
             A.stepq_intb_decode_step(self.cfg, self.bits, layer, self.pool, slots, q, k, v, beta,
                                      gate, y)

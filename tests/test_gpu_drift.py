@@ -71,3 +71,21 @@ def test_drift_run_short(torch):
     bpv = {n: v["bits_per_value"] for n, v in res["variants"].items()}
     assert 6.0 < bpv["stepq6"] < 6.6 and 4.0 < bpv["stepq4"] < 4.6
     assert 8.0 < bpv["int8"] < 8.2 and 4.0 < bpv["int4"] < 4.2
+
+
+def test_drift_ablations_short(torch):
+    """The component ablations of Sec. 5.4 run free for 32 steps: finite errors,
+    6-bit below 4-bit for each ablation, and storage near the nominal width."""
+    res = drift.run(steps=32, every=32, batch=4, warmup=8, variants=tuple(drift.ABLATIONS),
+                    calib=dict(seqs=2, steps=32))
+    last = res["records"][-1]
+    for name in drift.ABLATIONS:
+        e = last[name]["window_rms"]
+        assert math.isfinite(e) and 0.0 < e < 1.0, (name, e)
+    for a in ("spatial", "temporal", "temporal{}_nopiv", "stepq{}_nopiv"):
+        n6, n4 = (a.format(6), a.format(4)) if "{}" in a else (a + "6", a + "4")
+        assert last[n6]["window_rms"] < last[n4]["window_rms"]
+    bpv = {n: v["bits_per_value"] for n, v in res["variants"].items()}
+    for n, b in bpv.items():
+        nominal = 6 if "6" in n else 4
+        assert nominal < b < nominal + 0.6, (n, b)

@@ -149,6 +149,38 @@ def test_fp32_exact_read_decode(torch, name):
     assert A.stepq_device_error() == 0
 
 
+@pytest.mark.parametrize("name,kw", [("gqa", dict(n_pivots=3)), ("channel", {})])
+def test_temporal_codec(torch, name, kw):
+    """"Temporal only" ablation codec (Sec. 5.4): the plan's widths and FP16
+    pivots with the rowwise quantizer of App. B.5; pack is byte-exact against the
+    oracle and unpack reproduces the oracle's decode exactly."""
+    wl = W.WORKLOADS[name].replace(**kw)
+    cfg, plan, oplan, _ = plans(wl)
+    B = 8
+    slots = _slots(wl, B)
+    stride = A.stepq_temporal_slot_bytes(plan)
+    rb = oplan.layer_row_bits(0)
+    hb = [O.temporal_head_bytes(rb[h]) for h in range(wl.hv)]
+    off = np.concatenate([[0], np.cumsum(hb)])
+    S = W.random_states(wl, B * wl.hv).reshape(B, wl.hv, 128, 128)
+    pool_o = np.zeros(wl.pool_slots * stride, np.uint8)
+    ref = np.zeros_like(S)
+    for b in range(B):
+        for h in range(wl.hv):
+            base = int(slots[b]) * stride + int(off[h])
+            pool_o[base:base + hb[h]] = O.temporal_encode_head(S[b, h], rb[h])
+            ref[b, h] = O.temporal_decode_head(pool_o[base:base + hb[h]], rb[h])
+    assert (rb == 16).any()
+    S_d, slots_d = to_dev(S, slots)
+    pool_d = torch.zeros(wl.pool_slots * stride, dtype=torch.uint8, device="cuda")
+    A.stepq_temporal_quantize_pool(plan, 0, S_d, slots_d, pool_d)
+    assert np.array_equal(pool_d.cpu().numpy(), pool_o)
+    out = torch.empty_like(S_d)
+    A.stepq_temporal_dequantize_pool(plan, 0, pool_d, slots_d, out)
+    assert np.array_equal(out.cpu().numpy(), ref)
+    assert A.stepq_device_error() == 0
+
+
 @pytest.mark.parametrize("bits,name", [(8, "gqa"), (4, "channel"), (6, "gqa"), (6, "channel")])
 def test_intb_decode(torch, bits, name):
     """Uniform rowwise-absmax INT-b state (App. B.5), teacher-forced for 3 steps."""

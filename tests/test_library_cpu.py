@@ -83,6 +83,20 @@ def test_paper_shape_plan_bytes():
     assert plan.slot_stride == 29_999_104
 
 
+@pytest.mark.parametrize("name,kw", [("gqa", dict(n_pivots=3)), ("channel", {}), ("pool", dict(layers=2))])
+def test_temporal_slot_bytes(oracle, name, kw):
+    """"Temporal only" layout (Sec. 5.4): per head s[128] fp16 plus 16 b_i bytes per
+    row at the plan's widths (pivots 256 B), heads in (layer, head) order."""
+    wl = W.WORKLOADS[name].replace(**kw)
+    st = _stats(oracle, wl, seqs=1, steps=16)
+    oplan = oracle.plan_from_stats(wl, st)
+    cfg = A.Config.from_workload(wl)
+    plan = A.stepq_fit_scales(cfg, st.omega, st.mean_log_ret, st.dist, st.pivot)
+    total = sum(oracle.temporal_head_bytes(rb) for l in range(wl.layers)
+                for rb in oplan.layer_row_bits(l))
+    assert A.stepq_temporal_slot_bytes(plan) == (total + 255) // 256 * 256
+
+
 def test_argument_errors_before_launch():
     L = _lib.lib()
     cfg = A.Config(n_layers=1, n_key_heads=4, n_value_heads=4).c()
