@@ -8,14 +8,19 @@ The paper's workloads (Qwen3.8-27B / Kimi-Linear traces on WikiText-2 and C4) ar
 not available; these generators stand in for them with the shapes of the paper's
 hybrid models (d_k = d_v = 128, Sec. 2.1 and Table `config`) and the value
 structure it reports: scalar per-head gates for GDN, per-key-channel gates for
-KDA (Sec. 2.1), long-lived heads (Sec. 3.1) and per-key-row magnitude spread
-(Sec. 4.2).
+KDA (Sec. 2.1), long-lived heads (Sec. 3.1) and magnitude outliers along both
+key rows and value columns (Sec. 4.2, App. E): fixed lognormal key-channel and
+value-channel scales, sized so that the states' median max-to-median RMS
+contrasts match the ones the paper measures (about 10x rows / 19x columns for
+the GDN model, 13x / 5x for KDA).
 
 Recipe (every draw comes from numpy's PCG64 seeded by a SeedSequence over
 (seed, stream, step, layer), so any step of any layer can be drawn alone):
 
-* q, v ~ N(0, 1); k = n / ||n|| per key head, n ~ N(0, 1) scaled channel-wise by
-  fixed lognormal(0, 1) factors for the channel-gate workloads.
+* q ~ N(0, 1); k = n / ||n|| per key head, n ~ N(0, 1) scaled channel-wise by
+  fixed lognormal(0, k_sigma) factors per (layer, key head, channel);
+  v ~ N(0, 1) scaled by fixed lognormal(0, v_sigma) factors per (layer, value
+  head, channel).
 * beta = sigmoid(N(0, 1)) per (slot, value head).
 * scalar gate alpha ~ U(lo, hi) per (slot, value head, step); a fixed fraction of
   heads is "long-lived" with alpha ~ U(long_lo, long_hi).
@@ -63,7 +68,8 @@ class Workload:
     chan_lo: float = 0.80
     chan_hi: float = 0.999
     chan_jitter: float = 0.01
-    k_lognormal: bool = False
+    k_sigma: float = 0.0           # key-channel lognormal spread (row outliers)
+    v_sigma: float = 0.0           # value-channel lognormal spread (column outliers)
     calib_seqs: int = 8
     calib_steps: int = 256
     calib_every: int = 8
@@ -83,22 +89,31 @@ class Workload:
         return dataclasses.replace(self, **kw)
 
 
+# Channel spreads that give the states the paper's median max-to-median RMS
+# contrasts (App. E: GDN 10.3x key rows / 19.4x value columns; KDA 12.7x /
+# 5.4x), measured on snapshots of these recurrences from a zero state.
+GDN_K_SIGMA, GDN_V_SIGMA = 1.05, 1.12
+KDA_K_SIGMA, KDA_V_SIGMA = 1.10, 0.60
+
 # The five workloads: tiny decode, GQA decode, channel-gate decode, the 1024-slot
 # serving pool and the long-generation drift run.
 WORKLOADS = {
     "tiny": Workload("tiny", layers=1, hk=4, hv=4, batch=1, pool_slots=1, steps=64,
-                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0),
+                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0,
+                     k_sigma=GDN_K_SIGMA, v_sigma=GDN_V_SIGMA),
     "gqa": Workload("gqa", layers=1, hk=16, hv=32, batch=64, pool_slots=64, steps=256,
                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0,
-                    alpha_lo=0.85, alpha_hi=0.999, long_frac=0.25),
+                    alpha_lo=0.85, alpha_hi=0.999, long_frac=0.25,
+                    k_sigma=GDN_K_SIGMA, v_sigma=GDN_V_SIGMA),
     "channel": Workload("channel", layers=1, hk=32, hv=32, batch=256, pool_slots=256, steps=512,
                         gate="channel", nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=26,
-                        k_lognormal=True),
+                        k_sigma=KDA_K_SIGMA, v_sigma=KDA_V_SIGMA),
     "pool": Workload("pool", layers=16, hk=32, hv=32, batch=1024, pool_slots=1024, steps=128,
-                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=7),
+                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=7,
+                     k_sigma=GDN_K_SIGMA, v_sigma=GDN_V_SIGMA),
     "drift": Workload("drift", layers=4, hk=32, hv=32, batch=128, pool_slots=128, steps=8192,
                       gate="channel", nominal_bits=6, candidates=(4, 6, 8), n_pivots=102,
-                      k_lognormal=True),
+                      k_sigma=KDA_K_SIGMA, v_sigma=KDA_V_SIGMA),
 }
 
 
@@ -111,7 +126,8 @@ class ModelParams:
     """Fixed per-head properties of the synthetic model (shared by all streams)."""
     long_lived: np.ndarray      # [L][Hv] bool (scalar gate)
     chan_base: np.ndarray       # [L][Hv][DK] float64 (channel gate)
-    k_scale: np.ndarray         # [L][Hk][DK] float64 (1 unless lognormal)
+    k_scale: np.ndarray         # [L][Hk][DK] float64 (1 when k_sigma = 0)
+    v_scale: np.ndarray         # [L][Hv][DV] float64 (1 when v_sigma = 0)
 
 
 def model_params(wl: Workload) -> ModelParams:
@@ -121,11 +137,15 @@ def model_params(wl: Workload) -> ModelParams:
     for layer in range(wl.layers):
         long_lived[layer, g.permutation(wl.hv)[:n_long]] = True
     chan_base = g.uniform(wl.chan_lo, wl.chan_hi, size=(wl.layers, wl.hv, DK))
-    if wl.k_lognormal:
-        k_scale = g.lognormal(0.0, 1.0, size=(wl.layers, wl.hk, DK))
+    if wl.k_sigma > 0:
+        k_scale = g.lognormal(0.0, wl.k_sigma, size=(wl.layers, wl.hk, DK))
     else:
         k_scale = np.ones((wl.layers, wl.hk, DK))
-    return ModelParams(long_lived, chan_base, k_scale)
+    if wl.v_sigma > 0:
+        v_scale = g.lognormal(0.0, wl.v_sigma, size=(wl.layers, wl.hv, DV))
+    else:
+        v_scale = np.ones((wl.layers, wl.hv, DV))
+    return ModelParams(long_lived, chan_base, k_scale, v_scale)
 
 
 @dataclass
@@ -145,7 +165,7 @@ def step_inputs(wl: Workload, mp: ModelParams, stream: int, step: int, layer: in
     q = g.standard_normal((b, wl.hk, DK))
     n = g.standard_normal((b, wl.hk, DK)) * mp.k_scale[layer][None]
     k = n / np.linalg.norm(n, axis=-1, keepdims=True)
-    v = g.standard_normal((b, wl.hv, DV))
+    v = g.standard_normal((b, wl.hv, DV)) * mp.v_scale[layer][None]
     beta = 1.0 / (1.0 + np.exp(-g.standard_normal((b, wl.hv))))
     if wl.gate == "scalar":
         lo = np.where(mp.long_lived[layer], wl.long_lo, wl.alpha_lo)
@@ -182,7 +202,7 @@ def torch_step_inputs(wl: Workload, mp_dev: dict, step: int, layer: int, device,
 
     Used where the oracle never sees the values (timing runs). `mp_dev` holds the
     model params as device tensors: long_lived [L][Hv], chan_base [L][Hv][DK],
-    k_scale [L][Hk][DK].
+    k_scale [L][Hk][DK], v_scale [L][Hv][DV].
     """
     import torch
     g = torch.Generator(device=device)
@@ -192,7 +212,7 @@ def torch_step_inputs(wl: Workload, mp_dev: dict, step: int, layer: int, device,
     q = torch.randn((b, wl.hk, DK), generator=g, device=device, dtype=f)
     n = torch.randn((b, wl.hk, DK), generator=g, device=device, dtype=f) * mp_dev["k_scale"][layer][None]
     k = n / torch.linalg.vector_norm(n, dim=-1, keepdim=True)
-    v = torch.randn((b, wl.hv, DV), generator=g, device=device, dtype=f)
+    v = torch.randn((b, wl.hv, DV), generator=g, device=device, dtype=f) * mp_dev["v_scale"][layer][None]
     beta = torch.sigmoid(torch.randn((b, wl.hv), generator=g, device=device, dtype=f))
     if wl.gate == "scalar":
         ll = mp_dev["long_lived"][layer]
@@ -212,4 +232,5 @@ def model_params_torch(mp: ModelParams, device) -> dict:
         "long_lived": torch.as_tensor(mp.long_lived, device=device),
         "chan_base": torch.as_tensor(mp.chan_base, dtype=torch.float32, device=device),
         "k_scale": torch.as_tensor(mp.k_scale, dtype=torch.float32, device=device),
+        "v_scale": torch.as_tensor(mp.v_scale, dtype=torch.float32, device=device),
     }
