@@ -75,8 +75,17 @@ def test_prefill_empty_and_identity(torch):
 
 @pytest.mark.parametrize("name", ["gqa", "channel"])
 def test_prefill_boundary_packs_like_the_oracle(torch, name):
-    """Prefill from a stored state (unpack), then pack the boundary state: the
-    page matches the oracle's encoding of its own prefilled state."""
+    """Prefill from a stored state (unpack), then pack the boundary state.
+
+    The unpacked start is the oracle's decode exactly; the prefilled state is
+    within 1e-4 of the oracle's token-by-token recurrence; and the page packed
+    on the device matches the oracle's encoding of that same prefilled state
+    (the same-input parity bar: codes +-1 LSB on at most 1e-4 of elements).
+    The page is not compared with the oracle's encoding of its own prefilled
+    state: the two states differ by fp32 rounding, and in low-magnitude rows
+    (the key-row and value-column outliers give them steps far below 1e-4 of
+    the state's maximum) that difference alone can move a code by several
+    levels."""
     wl = W.WORKLOADS[name]
     B, T = 4, 48
     cfg, plan, oplan, _ = plans(wl)
@@ -86,16 +95,19 @@ def test_prefill_boundary_packs_like_the_oracle(torch, name):
     S_start = O.pool_decode(oplan, pool_o, 0, slots).astype(np.float32)
     q, k, v, beta, gate = _tokens(wl, B, T)
     S_o, _ = _reference(S_start, q, k, v, beta, gate)
-    pool_ref = pool_o.copy()
-    O.pool_encode(oplan, pool_ref, 0, slots, S_o)
     (slots_d,) = to_dev(slots)
     pool_d = torch.from_numpy(pool_o).cuda()
     states = torch.empty((B, wl.hv, 128, 128), dtype=torch.float32, device="cuda")
     A.stepq_dequantize_pool(plan, 0, pool_d, slots_d, states)
+    assert np.array_equal(states.cpu().numpy(), S_start)
     q_d, k_d, v_d, b_d, g_d = to_dev(q, k, v, beta, gate)
     y_d = torch.empty((B, T, wl.hv, 128), dtype=torch.float32, device="cuda")
     A.stepq_prefill_fp32(cfg, states, q_d, k_d, v_d, b_d, g_d, y_d)
+    S_g = states.cpu().numpy()
+    assert np.abs(S_g - S_o).max() <= 1e-4 * np.abs(S_o).max()
     A.stepq_quantize_pool(plan, 0, states, slots_d, pool_d)
+    pool_ref = pool_o.copy()
+    O.pool_encode(oplan, pool_ref, 0, slots, S_g)
     t = Tally()
     compare_pools(t, pool_d.cpu().numpy(), pool_ref, oplan, 0, slots)
     print(name, t.summary())
