@@ -16,9 +16,10 @@
  *    max_i fp32(fp32(|X_ij| rho_i) / qmax_i)), then applies `fit_iters`
  *    fixed-code updates c_j = sum w_i^2 v_ij X_ij / sum w_i^2 v_ij^2 (App. C.1),
  *    a zero denominator keeping the current iterate, floor 2^-14, cap 65504;
- *  - "round to the nearest level" is round-half-to-even of the fp32 value
- *    t = fp32(fp32(X * rho_i) * gamma_j), rho_i = fp32(1/(r_i zs_i)),
- *    gamma_j = fp32(1/c_j): the decision is taken in the GPU tile's precision;
+ *  - "round to the nearest level" is round-half-to-even of the exact product
+ *    X'_ij * gamma_j of the fp32 row-normalised value X'_ij = fp32(X * rho_i)
+ *    and gamma_j = fp32(1/c_j), rho_i = fp32(1/(r_i zs_i)): one rounding, as a
+ *    fused multiply-add with 1.5 * 2^23 takes it in the GPU tile;
  *  - codes are stored offset-binary u = q + 2^(b-1), LSB-first per row.
  *
  * Page layout of one head (all pieces 16-byte multiples):
@@ -54,6 +55,9 @@ static double clampd(double x, double lo, double hi) { return x < lo ? lo : (x >
 
 /* fp32 product of two fp32 values (exact in fp64, rounded once) */
 static float mul32(float a, float b) { return (float)((double)a * (double)b); }
+/* Nearest integer (ties to even) to the exact product of two fp32 values: the
+ * product of two floats is exact in fp64, so there is a single rounding. */
+static double rne_prod(float a, float b) { return rint((double)a * (double)b); }
 
 size_t or_head_bytes(int unit_kind, const int8_t *rb)
 {
@@ -220,8 +224,7 @@ static void fit_head(const float *X, int unit_kind, const int8_t *rb, const floa
                 if (!in_fit[i])
                     continue;
                 int b = rb[i], qm = qmax_of(b);
-                float t = mul32(mul32(X[i * OR_D + j], rho[i]), gamma);
-                double qv = clampd(rint((double)t), -qm, qm);
+                double qv = clampd(rne_prod(mul32(X[i * OR_D + j], rho[i]), gamma), -qm, qm);
                 if (z_last)
                     z_last[i * OR_D + j] = (int8_t)qv;
                 double v = r[i] * (double)zs_of(unit_kind, b) * qv;      /* v_ij = r_i z_ij */
@@ -279,8 +282,7 @@ void or_encode_head(const float *X, int unit_kind, const int8_t *rb, const float
                 put_u16(stream + pos / 8, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
                 continue;
             }
-            float t = mul32(mul32(X[i * OR_D + j], rho[i]), gamma[j]);
-            int qv = (int)clampd(rint((double)t), -qm, qm);
+            int qv = (int)clampd(rne_prod(mul32(X[i * OR_D + j], rho[i]), gamma[j]), -qm, qm);
             put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1))));
         }
     }
