@@ -243,8 +243,8 @@ __device__ __forceinline__ void abs_row_sums(const uint64_t (&x)[4], float &lo, 
 }
 
 // Least-squares sums of the thread's columns: n_j += alpha_i z_ij X'_ij and
-// d_j += alpha_i z_ij^2 with z_ij = rne(X'_ij / c_j), clamped to +-qmax when
-// CLIP (App. C.1).
+// d_j += alpha_i z_ij^2 with z_ij = rne(X'_ij gamma_j) (one rounding of the
+// exact product), clamped to +-qmax when CLIP (App. C.1).
 template <int B, bool CLIP>
 __device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_t (&x2)[8][4],
                                         const uint64_t (&g)[4], uint64_t (&n)[4], uint64_t (&d)[4]) {
@@ -260,7 +260,7 @@ __device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_
             const uint64_t al = h ? ahi : alo;
 #pragma unroll
             for (int c = 0; c < 4; c++) {
-                uint64_t q = fadd2(fadd2(fmul2(x2[m][c], g[c]), M2), nM2);
+                uint64_t q = fadd2(ffma2(x2[m][c], g[c], M2), nM2);   // rne of the exact product
                 if (CLIP) q = clamp2(q, fqm);
                 const uint64_t aq = fmul2(al, q);
                 n[c] = ffma2(aq, x2[m][c], n[c]);
@@ -270,22 +270,23 @@ __device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_
     }
 }
 
-// Final codes q_ij = rne(X'_ij / c_j) with the stored scales (clamped when
+// Final codes q_ij = rne(X'_ij gamma_j) with the stored scales (clamped when
 // CLIP), packed into the page chunks.
 template <int B, bool CLIP>
 __device__ __forceinline__ void final_codes(const T &t, const Smem &S, uint8_t *page,
                                             const uint64_t (&x2)[8][4]) {
     constexpr float fqm = (float)((1 << (B - 1)) - 1);
-    const uint64_t MB = f2s(kMagic + (float)(1 << (B - 1)));
+    constexpr float fmb = kMagic + (float)(1 << (B - 1));
+    const uint64_t MB = f2s(fmb), LO = f2s(fmb - fqm), HI = f2s(fmb + fqm);
 #pragma unroll
     for (int c = 0; c < 4; c++) {
         const uint64_t gc = col_pair(S.colG, t.col(c));
         uint32_t f[16];
 #pragma unroll
         for (int m = 0; m < 8; m++) {
-            uint64_t tq = fmul2(x2[m][c], gc);
-            if (CLIP) tq = clamp2(tq, fqm);
-            const uint64_t uu = fadd2(tq, MB);          // bits: 0x4B400000 | (q + 2^(B-1))
+            // one rounding of the exact product, then the clamp on the biased code
+            uint64_t uu = ffma2(x2[m][c], gc, MB);      // bits: 0x4B400000 | (q + 2^(B-1))
+            if (CLIP) uu = clamp2r(uu, LO, HI);
             f[2 * m] = (uint32_t)uu;
             f[2 * m + 1] = (uint32_t)(uu >> 32);
         }

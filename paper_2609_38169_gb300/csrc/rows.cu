@@ -243,13 +243,18 @@ __device__ __forceinline__ void store_pair(const T &t, const Smem &S, uint8_t *p
     const int b0 = (int)((inf.x >> 16) & 0xFFu), b1 = (int)((inf.z >> 16) & 0xFFu);
     uint8_t *r0 = page + (inf.x & 0xFFFFu), *r1 = page + (inf.z & 0xFFFFu);
     const uint64_t mb = row_pair(S.rMb, t, m);
-    const uint64_t qm = CLIP ? row_pair(S.rQm, t, m) : 0;
+    uint64_t lo = 0, hi = 0;
+    if (CLIP) {
+        const uint64_t qm = row_pair(S.rQm, t, m);
+        lo = f2(f2lo(mb) - f2lo(qm), f2hi(mb) - f2hi(qm));
+        hi = f2(f2lo(mb) + f2lo(qm), f2hi(mb) + f2hi(qm));
+    }
     uint32_t f[2][4];
 #pragma unroll
     for (int c = 0; c < 4; c++) {
-        uint64_t tq = fmul2(x[c], gd[c]);
-        if (CLIP) tq = clamp2p(tq, qm);
-        const uint64_t uu = fadd2(tq, mb);              // bits: 0x4B400000 | (q + 2^(b-1))
+        // one rounding of the exact product, then the clamp on the biased code
+        uint64_t uu = ffma2(x[c], gd[c], mb);           // bits: 0x4B400000 | (q + 2^(b-1))
+        if (CLIP) uu = clamp2r(uu, lo, hi);
         f[0][c] = (uint32_t)uu;
         f[1][c] = (uint32_t)(uu >> 32);
     }
@@ -284,7 +289,7 @@ __device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_
             const uint64_t al = h ? ahi : alo;
 #pragma unroll
             for (int c = 0; c < 4; c++) {
-                uint64_t q = fadd2(fadd2(fmul2(x2[m][c], g[c]), M2), nM2);
+                uint64_t q = fadd2(ffma2(x2[m][c], g[c], M2), nM2);   // rne of the exact product
                 if (CLIP) q = clamp2p(q, h ? qhi : qlo);
                 const uint64_t aq = fmul2(al, q);
                 n[c] = ffma2(aq, x2[m][c], n[c]);

@@ -8,14 +8,16 @@
 //
 // Numerical contract (shared with the CPU oracle, which restates it in fp64):
 // the tile X is fp32; r_i = fp16(clamp(sqrt(m_i) * w_i^(-1/2), 2^-14, 65504));
-// rho_i = fp32(1/(r_i zs_i)); every code decision is rint(fp32(fp32(X rho_i)
-// gamma_j)) with gamma_j = fp32(1/c_j); c is fitted from the clip-free start
+// rho_i = fp32(1/(r_i zs_i)); every code decision is the nearest integer to the
+// exact product fp32(X rho_i) gamma_j with gamma_j = fp32(1/c_j) (rne_prod);
+// c is fitted from the clip-free start
 // max_i fp32(fp32(|X_ij| rho_i) / qmax_i) by `fit_iters` fixed-code
 // least-squares updates.
 #include <cstdio>
 
 #include "device.cuh"
 #include "internal.h"
+#include "tile.cuh"
 
 namespace stepq {
 
@@ -125,8 +127,7 @@ __device__ __forceinline__ void fit_scales(const Lane &L, const TileSmem &S, con
             const float w2 = S.w2[L.row(t)], rz = f.rr[t] * f.zsv[t], lim = (float)f.qm[t];
 #pragma unroll
             for (int j = 0; j < 16; j++) {
-                const float tq = __fmul_rn(__fmul_rn(x[t][j], f.rho[t]), g[j]);
-                const float qv = fminf(fmaxf(rintf(tq), -lim), lim);
+                const float qv = fminf(fmaxf(rne_prod(__fmul_rn(x[t][j], f.rho[t]), g[j]), -lim), lim);
                 const float v = rz * qv;                      // v_ij = r_i z_ij
                 acc[0][j] += w2 * (v * x[t][j]);
                 acc[1][j] += w2 * (v * v);
@@ -170,7 +171,7 @@ __device__ __forceinline__ void pack_codes(const Lane &L, const TileSmem &S, con
         int q[16];
 #pragma unroll
         for (int j = 0; j < 16; j++)
-            q[j] = (int)fminf(fmaxf(rintf(__fmul_rn(__fmul_rn(x[t][j], f.rho[t]), g[j])), -lim), lim);
+            q[j] = (int)fminf(fmaxf(rne_prod(__fmul_rn(x[t][j], f.rho[t]), g[j]), -lim), lim);
         store_codes16(row, f.bits[t], L.cg, q);
     }
     __syncthreads();
@@ -358,7 +359,7 @@ __global__ void __launch_bounds__(kThreads, 2) distortion_kernel(DistArgs a) {
 #pragma unroll
                 for (int j = 0; j < 16; j++) {
                     const float cj = S.col[L.col0() + j], gj = S.col[128 + L.col0() + j];
-                    const float qv = fminf(fmaxf(rintf(__fmul_rn(__fmul_rn(x[t][j], f.rho[t]), gj)), -lim), lim);
+                    const float qv = fminf(fmaxf(rne_prod(__fmul_rn(x[t][j], f.rho[t]), gj), -lim), lim);
                     const float rec = __fmul_rn(f.rr[t] * cj, f.zsv[t] * qv);
                     const float d = rec - x[t][j];
                     e += d * d;

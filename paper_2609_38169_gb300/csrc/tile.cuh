@@ -18,6 +18,18 @@ __device__ __forceinline__ uint64_t clamp2(uint64_t v, float lim) {
     return f2(fminf(fmaxf(f2lo(v), -lim), lim), fminf(fmaxf(f2hi(v), -lim), lim));
 }
 
+// Clamp of a pair to [lo, hi] per half (used on magic-biased codes).
+__device__ __forceinline__ uint64_t clamp2r(uint64_t v, uint64_t lo, uint64_t hi) {
+    return f2(fminf(fmaxf(f2lo(v), f2lo(lo)), f2lo(hi)), fminf(fmaxf(f2hi(v), f2hi(lo)), f2hi(hi)));
+}
+
+// Nearest integer (ties to even) of the exact product a * b for |a b| < 2^22:
+// one fused multiply-add with 1.5 * 2^23 rounds it once. Larger products come
+// out within a few units of a b, which every caller clamps to +-qmax anyway.
+__device__ __forceinline__ float rne_prod(float a, float b) {
+    return __fmaf_rn(a, b, 12582912.0f) - 12582912.0f;
+}
+
 // Sum of 16 per-row partials over the 32 lanes of a warp (reduce-scatter): lane
 // l returns the full sum of row 8*b4 + 4*b3 + 2*b2 + b1 (b_k = bit k of l).
 __device__ __forceinline__ float warp_row_sums(float (&v)[16], int l, int &row_out) {
