@@ -187,6 +187,32 @@ stepq_status stepq_prefill_fp32(const stepq_config *cfg, int B, int T, float *st
                                 const float *beta, const float *gate, float *y,
                                 stepq_stream_t stream);
 
+/* The decode step split in two for a side stream (Sec. 4.4, App. F.1: after the
+ * readout, scale fitting and packed writeback run on a separate CUDA stream
+ * while later layers process the token; writeback completes before the next
+ * recurrent step reads the state). Head-unit (scalar-gate) plans only;
+ * row-unit plans return STEPQ_ERR_UNSUPPORTED.
+ *
+ * stepq_decode_readout: App. C.3 steps 1-3 of stepq_decode_step: reconstruct,
+ *   Delta update, readout. Writes y [B][Hv][128] and delta [B][Hv][128]
+ *   (delta_j = v_j - k^T D S_hat, device fp32, 16-byte aligned) and leaves the
+ *   pages unchanged. y is bit-identical to stepq_decode_step's.
+ * stepq_decode_writeback: steps 4-7 in place: rebuilds the updated tile from
+ *   the unchanged page, k, beta, gate and the readout's delta, refits and
+ *   packs it. The page is byte-identical to the one stepq_decode_step writes.
+ *   Order it after the readout of the same (layer, slots) (an event across
+ *   streams) and before the next step that reads those pages.
+ * Arguments and errors otherwise as for stepq_decode_step. */
+stepq_status stepq_decode_readout(const stepq_plan *plan, int layer, const void *pool,
+                                  int pool_slots, const int32_t *slots, int B, const float *q,
+                                  const float *k, const float *v, const float *beta,
+                                  const float *gate, float *y, float *delta,
+                                  stepq_stream_t stream);
+stepq_status stepq_decode_writeback(const stepq_plan *plan, int layer, void *pool, int pool_slots,
+                                    const int32_t *slots, int B, const float *k,
+                                    const float *beta, const float *gate, const float *delta,
+                                    stepq_stream_t stream);
+
 /* --------------------------------------------------- comparison kernels (same build)
  * FP32-state decode (the serving default the paper compares against, Sec. 5.1):
  * pool: device fp32 [pool_slots][L][Hv][128][128]; the step updates the layer's
@@ -198,7 +224,7 @@ stepq_status stepq_fp32_decode_step(const stepq_config *cfg, int layer, float *p
                                     const float *gate, float *y, stepq_stream_t stream);
 
 /* The exact-read counterpart of stepq_fp32_decode_step used by the feedback
- * experiment of App. B.4 ("exact-read oracle"): the retrieval reads the
+ * experiment of App. B.1 ("exact-read oracle"): the retrieval reads the
  * reference states, u = k^T D S_ref with S_ref from read_pool (same layout as
  * pool, not modified), while the update writes D S + beta k (v - u)^T into
  * pool. A state error E = S - S_ref then evolves as D E, without the Delta

@@ -172,7 +172,7 @@ def delta_batch(S, q, k, v, beta, gate):
 
 
 def delta_step_read(S, S_ref, q, k, v, beta, gate):
-    """Exact-read step of one head (App. B.4): the Delta residual reads the
+    """Exact-read step of one head (App. B.1): the Delta residual reads the
     reference state, u = k^T D S_ref; returns (S_new, y)."""
     S = _f32(S).copy()
     gate = _f32(np.atleast_1d(gate))

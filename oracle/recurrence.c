@@ -64,7 +64,7 @@ void or_delta_batch_f32(int n, int Hk, int Hv, int gate_per_row, float *S,
         }
 }
 
-/* The exact-read step of the feedback experiment (App. B.4): only the state
+/* The exact-read step of the feedback experiment (App. B.1): only the state
  * inside the Delta residual is replaced by the reference state S_ref,
  *   S_t = D_t S_{t-1} + beta_t k_t (v_t^T - k_t^T D_t S_ref_{t-1}),
  * so that S_t - S_ref_t = D_t (S_{t-1} - S_ref_{t-1}). S is updated in place;

@@ -39,6 +39,8 @@ SIGNATURES = {
     "stepq_plan_destroy": (None, [P]),
     "stepq_quantize_pool": (I, [P, I, P, P, I, P, I, P]),
     "stepq_dequantize_pool": (I, [P, I, P, I, P, I, P, P]),
+    "stepq_decode_readout": (I, [P, I, P, I, P, I, P, P, P, P, P, P, P, P]),
+    "stepq_decode_writeback": (I, [P, I, P, I, P, I, P, P, P, P, P]),
     "stepq_temporal_slot_bytes": (SZ, [P]),
     "stepq_temporal_quantize_pool": (I, [P, I, P, P, I, P, I, P]),
     "stepq_temporal_dequantize_pool": (I, [P, I, P, I, P, I, P, P]),

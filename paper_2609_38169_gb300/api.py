@@ -242,6 +242,31 @@ def stepq_decode_step(plan: Plan, layer: int, pool, slots, q, k, v, beta, gate, 
           "stepq_decode_step")
 
 
+def stepq_decode_readout(plan: Plan, layer: int, pool, slots, q, k, v, beta, gate, y, delta,
+                         pool_slots=None, stream=None):
+    import torch
+    f = torch.float32
+    check(_lib.lib().stepq_decode_readout(plan.handle, layer, _dev_ptr(pool),
+                                          _pool_slots(pool, plan.slot_stride, pool_slots),
+                                          _dev_ptr(slots, torch.int32), slots.numel(),
+                                          _dev_ptr(q, f), _dev_ptr(k, f), _dev_ptr(v, f),
+                                          _dev_ptr(beta, f), _dev_ptr(gate, f), _dev_ptr(y, f),
+                                          _dev_ptr(delta, f), _stream(stream)),
+          "stepq_decode_readout")
+
+
+def stepq_decode_writeback(plan: Plan, layer: int, pool, slots, k, beta, gate, delta,
+                           pool_slots=None, stream=None):
+    import torch
+    f = torch.float32
+    check(_lib.lib().stepq_decode_writeback(plan.handle, layer, _dev_ptr(pool),
+                                            _pool_slots(pool, plan.slot_stride, pool_slots),
+                                            _dev_ptr(slots, torch.int32), slots.numel(),
+                                            _dev_ptr(k, f), _dev_ptr(beta, f), _dev_ptr(gate, f),
+                                            _dev_ptr(delta, f), _stream(stream)),
+          "stepq_decode_writeback")
+
+
 def stepq_fp32_decode_step(cfg: Config, layer: int, pool, slots, q, k, v, beta, gate, y,
                            pool_slots=None, stream=None):
     import torch

@@ -127,6 +127,39 @@ extern "C" stepq_status stepq_decode_step(const stepq_plan *p, int layer, void *
                          (cudaStream_t)stream);
 }
 
+extern "C" stepq_status stepq_decode_readout(const stepq_plan *p, int layer, const void *pool,
+                                             int pool_slots, const int32_t *slots, int B,
+                                             const float *q, const float *k, const float *v,
+                                             const float *beta, const float *gate, float *y,
+                                             float *delta, stepq_stream_t stream) {
+    stepq_status st = check_plan_call(p, layer, false, pool, pool_slots, slots, B);
+    if (st != STEPQ_OK) return st;
+    if (p->cfg.gate_kind == STEPQ_GATE_CHANNEL) return STEPQ_ERR_UNSUPPORTED;
+    if (!v || !y || !delta) return STEPQ_ERR_ARG;
+    if ((st = check_inputs(&p->cfg, q, k, v, beta, gate, y)) != STEPQ_OK) return st;
+    if (!aligned(delta, 16)) return STEPQ_ERR_ALIGN;
+    if (B == 0) return STEPQ_OK;
+    return launch_decode_heads_mode(p, layer, (uint8_t *)pool, pool_slots, slots, B, q, k, v, beta,
+                                    gate, y, delta, 1, (cudaStream_t)stream);
+}
+
+extern "C" stepq_status stepq_decode_writeback(const stepq_plan *p, int layer, void *pool,
+                                               int pool_slots, const int32_t *slots, int B,
+                                               const float *k, const float *beta,
+                                               const float *gate, const float *delta,
+                                               stepq_stream_t stream) {
+    stepq_status st = check_plan_call(p, layer, false, pool, pool_slots, slots, B);
+    if (st != STEPQ_OK) return st;
+    if (p->cfg.gate_kind == STEPQ_GATE_CHANNEL) return STEPQ_ERR_UNSUPPORTED;
+    if (!k || !beta || !gate || !delta) return STEPQ_ERR_ARG;
+    if (!aligned(k, 16) || !aligned(delta, 16) || !aligned(beta, 4) || !aligned(gate, 4))
+        return STEPQ_ERR_ALIGN;
+    if (B == 0) return STEPQ_OK;
+    return launch_decode_heads_mode(p, layer, (uint8_t *)pool, pool_slots, slots, B, nullptr, k,
+                                    nullptr, beta, gate, nullptr, (float *)delta, 2,
+                                    (cudaStream_t)stream);
+}
+
 extern "C" stepq_status stepq_fp32_decode_step(const stepq_config *cfg, int layer, float *pool,
                                                int pool_slots, const int32_t *slots, int B,
                                                const float *q, const float *k, const float *v,

@@ -474,6 +474,11 @@ __device__ __forceinline__ void load_tile(const T &t, const uint8_t *page, uint6
 }
 
 // ------------------------------------------------------------------ decode
+// Kernel modes: the fused step, and the two halves of the side-stream split
+// (the readout returns y and delta and leaves the page as it is; the writeback
+// rebuilds the updated tile from the old page and delta, refits and packs it).
+enum : int { kFused = 0, kReadout = 1, kWriteback = 2 };
+
 struct DecodeArgs {
     uint8_t *pool;
     uint64_t stride;
@@ -483,6 +488,7 @@ struct DecodeArgs {
     LayerTables tab;
     const float *q, *k, *v, *beta, *gate;
     float *y;
+    float *delta;              // readout: delta_j out; writeback: delta_j in
     unsigned int *err;
     int n_stages;
     uint32_t page_region, stage_bytes;
@@ -490,19 +496,25 @@ struct DecodeArgs {
 };
 
 // Producer: start the copies of the item (head h, batch entry b, a valid slot)
-// into stage s.
+// into stage s. The writeback loads delta into the v slot and needs no q; the
+// readout needs no w2, wis.
+template <int MODE>
 __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s) {
     uint64_t *bar = &S.bars[s];
     Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
     const uint32_t nb = S.hbytes[h];
     const int hk = S.hkey[h];
-    mbar_arrive_tx(bar, nb + kVecBytes);
+    constexpr uint32_t vec = MODE == kFused ? kVecBytes : 4 * 512 - (MODE == kReadout ? 512 : 0);
+    mbar_arrive_tx(bar, nb + vec);
     bulk_load(st.page, a.pool + (uint64_t)slot * a.stride + S.hoff[h], nb, bar);
-    bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
+    if (MODE != kWriteback) bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
     bulk_load(st.k, a.k + ((size_t)b * a.Hk + hk) * 128, 512, bar);
-    bulk_load(st.v, a.v + ((size_t)b * a.Hv + h) * 128, 512, bar);
-    bulk_load(st.w2, a.tab.w2 + (size_t)h * 128, 512, bar);
-    bulk_load(st.wis, a.tab.wis + (size_t)h * 128, 512, bar);
+    if (MODE != kWriteback) bulk_load(st.v, a.v + ((size_t)b * a.Hv + h) * 128, 512, bar);
+    else bulk_load(st.v, a.delta + ((size_t)b * a.Hv + h) * 128, 512, bar);
+    if (MODE != kReadout) {
+        bulk_load(st.w2, a.tab.w2 + (size_t)h * 128, 512, bar);
+        bulk_load(st.wis, a.tab.wis + (size_t)h * 128, 512, bar);
+    }
 }
 
 // One decode step of one head page staged in shared memory (width B).
@@ -513,10 +525,15 @@ __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h,
 //
 // With a_i = alpha r_i (> 0) and Z_ij = c_j q_ij + (beta k_i / a_i) delta_j the
 // update is X_ij = a_i Z_ij: one fma per element instead of two.
-template <int B, class Refill>
+//
+// MODE kReadout stops after the readout: it writes y and delta (delta_out) and
+// leaves the page untouched. MODE kWriteback takes delta from the stage (the
+// readout's, bit for bit), rebuilds Z exactly as the fused step does, and runs
+// steps 4-6; its y is not computed.
+template <int B, int MODE, class Refill>
 __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Stage &st, float alpha,
-                                            float beta, float *y_out, int fit_iters, bool ok,
-                                            const Refill &refill) {
+                                            float beta, float *y_out, float *delta_out, int fit_iters,
+                                            bool ok, const Refill &refill) {
     const uint16_t *page_r = (const uint16_t *)st.page;
     // Row constants of the warp's band (warp-local).
     if (t.l < 16) {
@@ -525,13 +542,41 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         const float ki = st.k[i];
         S.rKap[i] = ki * a;
         S.rBkp[i] = __fdividef(beta * ki, a);          // within 2 ulp: Z carries rounding anyway
-        S.rQa[i] = st.q[i] * a;
+        if (MODE != kWriteback) S.rQa[i] = st.q[i] * a;
         S.rA[i] = a;
     }
-    if (t.tid < 128) S.colM[t.tid] = 0u;
+    if (MODE != kReadout && t.tid < 128) S.colM[t.tid] = 0u;
     uint64_t x2[8][4];
     load_tile<B>(t, st.page, x2);
     __syncwarp();
+    if constexpr (MODE == kWriteback) {
+        if (__syncthreads_or(!ok)) return false;
+        refill();
+        // Z = c q + (beta k / a) delta with the readout's delta; row sums of |Z|.
+        uint64_t dl[4];
+#pragma unroll
+        for (int c = 0; c < 4; c++) dl[c] = f2s(st.v[t.col(c)]);
+        float rs[16];
+#pragma unroll
+        for (int p = 0; p < 4; p++) {
+            uint64_t blo, bhi;
+            row_pairs(S.rBkp, t, p, blo, bhi);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                x2[2 * p][c] = ffma2(blo, dl[c], x2[2 * p][c]);
+                x2[2 * p + 1][c] = ffma2(bhi, dl[c], x2[2 * p + 1][c]);
+            }
+            abs_row_sums(x2[2 * p], rs[4 * p], rs[4 * p + 1]);
+            abs_row_sums(x2[2 * p + 1], rs[4 * p + 2], rs[4 * p + 3]);
+        }
+        if (B == kPivot) {
+            pack_pivot(t, st.page, x2, fmaxf(alpha, 1e-30f));
+            return true;
+        }
+        const float none[4] = {0.f, 0.f, 0.f, 0.f};
+        fit_pack<B>(t, S, st.page, st.w2, st.wis, true, x2, rs, none, false, nullptr, fit_iters);
+        return true;
+    }
     // Step 2a: retrieval u_j = sum_i k_i a_i (c_j q_ij).
     {
         uint64_t ua[4] = {0, 0, 0, 0}, ub[4] = {0, 0, 0, 0};
@@ -556,6 +601,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         for (int wv = 0; wv < 8; wv++) s += S.red[wv * 128 + t.tid];
         const float dl = st.v[t.tid] - s;                  // delta_j = v_j - u_j
         S.colD[t.tid] = make_float2(dl, dl);
+        if (MODE == kReadout) delta_out[t.tid] = dl;
     }
     refill();
     __syncthreads();
@@ -577,12 +623,14 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
             ya[c] = ffma2(qlo, x2[2 * p][c], ya[c]);
             yb[c] = ffma2(qhi, x2[2 * p + 1][c], yb[c]);
         }
-        abs_row_sums(x2[2 * p], rs[4 * p], rs[4 * p + 1]);
-        abs_row_sums(x2[2 * p + 1], rs[4 * p + 2], rs[4 * p + 3]);
+        if (MODE == kFused) {
+            abs_row_sums(x2[2 * p], rs[4 * p], rs[4 * p + 1]);
+            abs_row_sums(x2[2 * p + 1], rs[4 * p + 2], rs[4 * p + 3]);
+        }
     }
     const float yp[4] = {pair_sum(fadd2(ya[0], yb[0])), pair_sum(fadd2(ya[1], yb[1])),
                          pair_sum(fadd2(ya[2], yb[2])), pair_sum(fadd2(ya[3], yb[3]))};
-    if (B == kPivot) {
+    if (B == kPivot || MODE == kReadout) {
         const float v[1][4] = {{yp[0], yp[1], yp[2], yp[3]}};
         cols_to_red<1>(t, S.red, 2, v);
         __syncthreads();
@@ -593,7 +641,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
             for (int wv = 1; wv < 8; wv++) s += S.red[(2 * 8 + wv) * 128 + j];
             y_out[j] = s;
         }
-        pack_pivot(t, st.page, x2, fmaxf(alpha, 1e-30f));
+        if (MODE == kFused) pack_pivot(t, st.page, x2, fmaxf(alpha, 1e-30f));
         return true;
     }
     // Steps 4-6: refit and repack in place.
@@ -601,6 +649,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     return true;
 }
 
+template <int MODE>
 __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     const T t;
@@ -621,22 +670,25 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
     const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err};
     pipe::run(
         p, S.bars,
-        [&](int h, int b, int slot, int s) { issue(a, S, h, b, slot, s); },
+        [&](int h, int b, int slot, int s) { issue<MODE>(a, S, h, b, slot, s); },
         [&](int h, int b, int, int s, bool ok, const auto &refill) {
-            const float2 gb = make_float2(a.gate[(size_t)b * a.Hv + h], a.beta[(size_t)b * a.Hv + h]);
+            const size_t u = (size_t)b * a.Hv + h;
+            const float2 gb = make_float2(a.gate[u], a.beta[u]);
             const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
-            float *y_out = a.y + ((size_t)b * a.Hv + h) * 128;
+            float *y_out = MODE == kWriteback ? nullptr : a.y + u * 128;
+            float *d_out = MODE == kReadout ? a.delta + u * 128 : nullptr;
             switch (S.hbits[h]) {
-            case 2: return decode_item<2>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
-            case 4: return decode_item<4>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
-            case 6: return decode_item<6>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
-            case 8: return decode_item<8>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
-            default: return decode_item<kPivot>(t, S, st, gb.x, gb.y, y_out, a.fit_iters, ok, refill);
+            case 2: return decode_item<2, MODE>(t, S, st, gb.x, gb.y, y_out, d_out, a.fit_iters, ok, refill);
+            case 4: return decode_item<4, MODE>(t, S, st, gb.x, gb.y, y_out, d_out, a.fit_iters, ok, refill);
+            case 6: return decode_item<6, MODE>(t, S, st, gb.x, gb.y, y_out, d_out, a.fit_iters, ok, refill);
+            case 8: return decode_item<8, MODE>(t, S, st, gb.x, gb.y, y_out, d_out, a.fit_iters, ok, refill);
+            default: return decode_item<kPivot, MODE>(t, S, st, gb.x, gb.y, y_out, d_out, a.fit_iters, ok, refill);
             }
         },
         [&](int h, int slot, int s) {
-            bulk_store(a.pool + (uint64_t)slot * a.stride + S.hoff[h],
-                       S.stages + (size_t)s * a.stage_bytes, S.hbytes[h]);
+            if (MODE != kReadout)
+                bulk_store(a.pool + (uint64_t)slot * a.stride + S.hoff[h],
+                           S.stages + (size_t)s * a.stage_bytes, S.hbytes[h]);
         });
 }
 
@@ -775,6 +827,14 @@ stepq_status launch_decode_heads(const stepq_plan *p, int layer, uint8_t *pool, 
                                  const int32_t *slots, int B, const float *q, const float *k,
                                  const float *v, const float *beta, const float *gate, float *y,
                                  cudaStream_t s) {
+    return launch_decode_heads_mode(p, layer, pool, pool_slots, slots, B, q, k, v, beta, gate, y,
+                                    nullptr, hk::kFused, s);
+}
+
+stepq_status launch_decode_heads_mode(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
+                                      const int32_t *slots, int B, const float *q, const float *k,
+                                      const float *v, const float *beta, const float *gate, float *y,
+                                      float *delta, int mode, cudaStream_t s) {
     const int Hv = p->cfg.n_value_heads;
     if (Hv > hk::kMaxHv) return STEPQ_ERR_UNSUPPORTED;
     uint32_t maxb = 0;
@@ -791,6 +851,7 @@ stepq_status launch_decode_heads(const stepq_plan *p, int layer, uint8_t *pool, 
     a.items = B * Hv;
     a.tab = p->layer(layer);
     a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
+    a.delta = delta;
     a.err = device_error_word();
     a.page_region = (maxb + 127) / 128 * 128;
     a.stage_bytes = a.page_region + hk::kVecBytes;
@@ -800,10 +861,15 @@ stepq_status launch_decode_heads(const stepq_plan *p, int layer, uint8_t *pool, 
     a.n_stages = stages;
     a.fit_iters = p->cfg.fit_iters;
     const int smem = hk::kOffStages + stages * (int)a.stage_bytes;
-    if (set_attr((const void *)hk::decode_heads_kernel, smem) != STEPQ_OK) return STEPQ_ERR_CUDA;
+    const void *fn = mode == hk::kReadout     ? (const void *)hk::decode_heads_kernel<hk::kReadout>
+                     : mode == hk::kWriteback ? (const void *)hk::decode_heads_kernel<hk::kWriteback>
+                                              : (const void *)hk::decode_heads_kernel<hk::kFused>;
+    if (set_attr(fn, smem) != STEPQ_OK) return STEPQ_ERR_CUDA;
     int grid = 2 * sm_count();
     if (grid > a.items) grid = a.items;
-    hk::decode_heads_kernel<<<grid, kThreads, smem, s>>>(a);
+    if (mode == hk::kReadout) hk::decode_heads_kernel<hk::kReadout><<<grid, kThreads, smem, s>>>(a);
+    else if (mode == hk::kWriteback) hk::decode_heads_kernel<hk::kWriteback><<<grid, kThreads, smem, s>>>(a);
+    else hk::decode_heads_kernel<hk::kFused><<<grid, kThreads, smem, s>>>(a);
     return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;
 }
 

@@ -109,6 +109,11 @@ stepq_status launch_decode_heads(const stepq_plan *p, int layer, uint8_t *pool, 
                                  const int32_t *slots, int B, const float *q, const float *k,
                                  const float *v, const float *beta, const float *gate, float *y,
                                  cudaStream_t s);
+// mode 0 fused, 1 readout (y and delta out, pages untouched), 2 writeback (delta in)
+stepq_status launch_decode_heads_mode(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
+                                      const int32_t *slots, int B, const float *q, const float *k,
+                                      const float *v, const float *beta, const float *gate, float *y,
+                                      float *delta, int mode, cudaStream_t s);
 stepq_status launch_quantize_heads(const stepq_plan *p, int layer, const float *states,
                                    size_t stride_b, const int32_t *slots, int B, uint8_t *pool,
                                    int pool_slots, cudaStream_t s);

@@ -1,4 +1,4 @@
-"""Single-injection feedback experiment (App. B.4).
+"""Single-injection feedback experiment (App. B.1).
 
 The FP32-state recurrence runs from a zero state. After `inject` updates its
 state is quantized once (uniform INT-b, App. B.5, or a STEPQuant plan) and

@@ -6,6 +6,7 @@ generators), resident on the device, and timed with CUDA events after warm-up.
 
     python -m paper_2609_38169_gb300.measure rows [--slots 1024] [--bits 6]
     python -m paper_2609_38169_gb300.measure prefill [--slots 128] [--tokens 512]
+    python -m paper_2609_38169_gb300.measure split [--slots 1024] [--layers 16]
 """
 from __future__ import annotations
 
@@ -106,6 +107,95 @@ def prefill(slots=128, tokens=512, name="gqa"):
                          "frac": 2 * fma * head_tokens / t / FP32_FMA_PEAK_FLOPS}}
 
 
+def split(slots=1024, layers=16):
+    """The serving pool's decode step fused and split (Sec. 4.4, App. F.1).
+
+    Per-launch times of one layer for the fused kernel, the readout and the
+    writeback; then one token through all layers three ways: fused launches on
+    one stream; readout and writeback on one stream; readout on the main
+    stream with each writeback on a side stream ordered by an event (the
+    paper's arrangement). For the side-stream form the time until the last
+    layer's y is ready on the main stream is reported beside the total."""
+    import torch
+    dev = torch.device("cuda")
+    wl = W.WORKLOADS["pool"].replace(layers=layers, batch=slots, pool_slots=slots)
+    cfg = A.Config.from_workload(wl)
+    st = A.calibrate(cfg, wl, dev, seqs=4, steps=64, device_inputs=True)
+    plan = A.stepq_fit_scales(cfg, st.omega, st.mean_log_ret, st.dist, st.pivot)
+    pool = A.alloc_pool(plan, slots, dev)
+    all_slots = torch.arange(slots, dtype=torch.int32, device=dev)
+    g = torch.Generator(device=dev)
+    g.manual_seed(11)
+    S = torch.empty((slots, 1, wl.hv, D, D), device=dev)
+    for layer in range(layers):
+        S.normal_(generator=g)
+        A.stepq_quantize_pool(plan, layer, S[:, 0], all_slots, pool)
+    del S
+    perm = torch.from_numpy(W.slot_permutation(wl)).to(dev)
+    mp = W.model_params_torch(W.model_params(wl), dev)
+    inp = [W.torch_step_inputs(wl, mp, 0, layer, dev) for layer in range(layers)]
+    y = torch.empty((layers, slots, wl.hv, D), device=dev)
+    delta = torch.empty_like(y)
+    units = slots * wl.hv
+    out = {"metric": "side-stream split of the decode step", "unit": "us",
+           "workload": f"pool: {layers} layers x {slots} slots x {wl.hv} heads, STEPQuant @6",
+           "per_launch_us": {}}
+    q, k, v, beta, gate = inp[0]
+    out["per_launch_us"]["fused"] = 1e6 * _timeit(
+        lambda: A.stepq_decode_step(plan, 0, pool, perm, q, k, v, beta, gate, y[0]))
+    out["per_launch_us"]["readout"] = 1e6 * _timeit(
+        lambda: A.stepq_decode_readout(plan, 0, pool, perm, q, k, v, beta, gate, y[0], delta[0]))
+    out["per_launch_us"]["writeback"] = 1e6 * _timeit(
+        lambda: A.stepq_decode_writeback(plan, 0, pool, perm, k, beta, gate, delta[0]))
+
+    main, side = torch.cuda.current_stream(), torch.cuda.Stream()
+
+    def fused():
+        for layer in range(layers):
+            q, k, v, beta, gate = inp[layer]
+            A.stepq_decode_step(plan, layer, pool, perm, q, k, v, beta, gate, y[layer])
+
+    def serial():
+        for layer in range(layers):
+            q, k, v, beta, gate = inp[layer]
+            A.stepq_decode_readout(plan, layer, pool, perm, q, k, v, beta, gate, y[layer], delta[layer])
+            A.stepq_decode_writeback(plan, layer, pool, perm, k, beta, gate, delta[layer])
+
+    def two_streams(marks):
+        marks[0].record(main)
+        for layer in range(layers):
+            q, k, v, beta, gate = inp[layer]
+            A.stepq_decode_readout(plan, layer, pool, perm, q, k, v, beta, gate, y[layer],
+                                   delta[layer], stream=main)
+            ready = torch.cuda.Event()
+            ready.record(main)
+            side.wait_event(ready)
+            A.stepq_decode_writeback(plan, layer, pool, perm, k, beta, gate, delta[layer], stream=side)
+        marks[1].record(main)                        # the last y is ready
+        done = torch.cuda.Event()
+        done.record(side)
+        main.wait_event(done)                        # writeback before the next token
+        marks[2].record(main)
+
+    n = 10
+    out["token_ms"] = {"fused": 1e3 * _timeit(fused, n=n), "split_one_stream": 1e3 * _timeit(serial, n=n)}
+    for _ in range(3):
+        two_streams([torch.cuda.Event(enable_timing=True) for _ in range(3)])
+    torch.cuda.synchronize()
+    to_y, total = [], []
+    for _ in range(n):
+        marks = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        two_streams(marks)
+        torch.cuda.synchronize()
+        to_y.append(marks[0].elapsed_time(marks[1]))
+        total.append(marks[0].elapsed_time(marks[2]))
+    out["token_ms"]["split_side_stream_last_y"] = sum(to_y) / n
+    out["token_ms"]["split_side_stream_total"] = sum(total) / n
+    out["head_updates_per_token"] = units * layers
+    assert A.stepq_device_error() == 0
+    return out
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     sub = ap.add_subparsers(dest="what", required=True)
@@ -116,9 +206,14 @@ def main(argv=None):
     p.add_argument("--slots", type=int, default=128)
     p.add_argument("--tokens", type=int, default=512)
     p.add_argument("--workload", default="gqa", choices=["gqa", "channel", "pool"])
+    sp = sub.add_parser("split")
+    sp.add_argument("--slots", type=int, default=1024)
+    sp.add_argument("--layers", type=int, default=16)
     args = ap.parse_args(argv)
     if args.what == "rows":
         res = rows(args.slots, args.bits)
+    elif args.what == "split":
+        res = split(args.slots, args.layers)
     else:
         res = prefill(args.slots, args.tokens, args.workload)
     print(json.dumps(res))

@@ -9,7 +9,7 @@ not available; these generators stand in for them with the shapes of the paper's
 hybrid models (d_k = d_v = 128, Sec. 2.1 and Table `config`) and the value
 structure it reports: scalar per-head gates for GDN, per-key-channel gates for
 KDA (Sec. 2.1), long-lived heads (Sec. 3.1) and magnitude outliers along both
-key rows and value columns (Sec. 4.2, App. E): fixed lognormal key-channel and
+key rows and value columns (Sec. 4.2, App. B.6): fixed lognormal key-channel and
 value-channel scales, sized so that the states' median max-to-median RMS
 contrasts match the ones the paper measures (about 10x rows / 19x columns for
 the GDN model, 13x / 5x for KDA).
@@ -90,7 +90,7 @@ class Workload:
 
 
 # Channel spreads that give the states the paper's median max-to-median RMS
-# contrasts (App. E: GDN 10.3x key rows / 19.4x value columns; KDA 12.7x /
+# contrasts (App. B.6: GDN 10.3x key rows / 19.4x value columns; KDA 12.7x /
 # 5.4x), measured on snapshots of these recurrences from a zero state.
 GDN_K_SIGMA, GDN_V_SIGMA = 1.05, 1.12
 KDA_K_SIGMA, KDA_V_SIGMA = 1.10, 0.60

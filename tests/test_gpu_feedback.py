@@ -1,4 +1,4 @@
-"""Single-injection feedback experiment (App. B.4) on the GPU against the oracle.
+"""Single-injection feedback experiment (App. B.1) on the GPU against the oracle.
 
 The device driver (`feedback.run`) and a plain oracle restatement of the same
 experiment take the same seeded inputs; their per-trajectory error sums for

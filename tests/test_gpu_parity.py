@@ -119,7 +119,7 @@ def test_fp32_state_decode(torch):
 
 @pytest.mark.parametrize("name", ["gqa", "channel"])
 def test_fp32_exact_read_decode(torch, name):
-    """Exact-read step of the feedback experiment (App. B.4): the residual reads
+    """Exact-read step of the feedback experiment (App. B.1): the residual reads
     a separate reference pool, which the kernel leaves untouched."""
     wl = W.WORKLOADS[name]
     cfg = A.Config.from_workload(wl)

@@ -113,6 +113,9 @@ def test_argument_errors_before_launch():
     assert L.stepq_fp32_exact_read_step(C.byref(cfg), 0, C.c_void_p(256), None, 1, C.c_void_p(256), 1,
                                         None, None, C.c_void_p(256), None, None, C.c_void_p(256),
                                         None) == 1
+    assert L.stepq_decode_readout(None, 0, None, 1, None, 1, None, None, None, None, None, None,
+                                  None, None) == 1
+    assert L.stepq_decode_writeback(None, 0, None, 1, None, 1, None, None, None, None, None) == 1
     assert L.stepq_intb_slot_bytes(C.byref(cfg), 3) == 0
     assert L.stepq_intb_slot_bytes(C.byref(cfg), 8) == (256 + 128 * 128) * 4
     assert L.stepq_intb_slot_bytes(C.byref(cfg), 6) == (256 + 128 * 96) * 4
@@ -157,7 +160,7 @@ def test_feedback_cli():
 def test_measure_cli():
     """The secondary-measurement module parses its subcommands (no device work)."""
     from paper_2609_38169_gb300 import measure
-    for argv in (["--help"], ["rows", "--help"], ["prefill", "--help"]):
+    for argv in (["--help"], ["rows", "--help"], ["prefill", "--help"], ["split", "--help"]):
         with pytest.raises(SystemExit) as e:
             measure.main(argv)
         assert e.value.code == 0

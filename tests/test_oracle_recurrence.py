@@ -73,7 +73,7 @@ def test_directional_contraction(oracle, rng):
 
 @pytest.mark.parametrize("per_row", [False, True])
 def test_exact_read_error_is_only_decayed(oracle, rng, per_row):
-    """App. B.4: with the residual reading the reference state, the path's error
+    """App. B.1: with the residual reading the reference state, the path's error
     evolves as E_t = D_t E_{t-1}, while the native step gives (I - beta k k^T) D E."""
     S_ref = (rng.standard_normal((D, D)) * np.exp(rng.normal(size=(D, 1)))).astype(np.float32)
     E = (1e-2 * rng.standard_normal((D, D)) * np.abs(S_ref).max()).astype(np.float32)

@@ -1,6 +1,6 @@
 """The synthetic input recipe against the state geometry the paper measures.
 
-App. E reports, for FP32 states reconstructed from native inputs, the median
+App. B.6 reports, for FP32 states reconstructed from native inputs, the median
 over snapshots of the maximum-to-median RMS contrast along key rows and along
 value columns: 10.3x and 19.4x for the GDN model (Qwen, positions 128 to
 2,048), 12.7x and 5.4x for KDA (Kimi-Linear, steps 128 to 512). The workload
