@@ -10,29 +10,29 @@
 //   w_t = beta_t (v_t - S_0^T g_t k_t - sum_{s<t} (k_s/g_s . g_t k_t) w_s),
 // i.e. (I + A) W = diag(beta) (V - K~ S_0) with K~ = G K, K^ = G^-1 K and
 // A_ts = beta_t (K~_t . K^_s) for s < t; the outputs are
-//   Y = Q~ S_0 + tril(Q~ K^T) W   (Q~ = G Q, lower triangle with the diagonal),
+//   Y = Q~ S_0 + Bm W,  Bm = tril(Q~ K^T) (Q~ = G Q, lower triangle with the diagonal),
 // and the state after the chunk is S_C = G_C S_0 + K_bar^T W, K_bar = K g_C / g.
 //
-// The two large products run on the tensor cores (tcgen05, kind::tf32) with
-// the state resident in tensor memory as S^T (lane j = value column, column i
-// = key row), in split precision: every fp32 operand is a TF32 head plus its
-// remainder, and a product is head*head + head*rest + rest*head (the rest*rest
-// term is below fp32 rounding of the accumulation), so the chunk keeps fp32
-// accuracy:
-//   P1  [K~ S_0 ; Q~ S_0]^T = S_0^T [K~ ; Q~]^T   M = 128 (j), N = 64, K = 128
-//   P2  S^T += W^T K_bar                            M = 128 (j), N = 128, K = 32
-// with A (S^T or W^T) in tensor memory and B ([K~ ; Q~] or K_bar^T) in shared
-// memory as K-major core matrices. The 32 x 32 products A and Q~ K^T, the
-// triangular solve (one value column per thread) and the readout
-// Y = Q~ S_0 + tril(Q~ K^T) W stay on the FMA pipe.
+// Every product runs on the tensor cores (tcgen05, kind::tf32) in split
+// precision: an fp32 operand is a TF32 head plus its remainder, and a product
+// is head*head + head*rest + rest*head (the rest*rest term is below fp32
+// rounding of the accumulation), which keeps fp32 accuracy. The state stays
+// in tensor memory as S^T (lane j = value column, column i = key row):
+//   P0  [K~ ; Q~] K^T        -> A, Bm      M = 128 (64 used), N = 32, K = 128, A, B in smem
+//   P1  S_0^T [K~ ; Q~]^T    -> [K~ S_0 ; Q~ S_0]^T    M = 128, N = 64, K = 128, A in tmem
+//   P2  S^T += W^T K_bar                               M = 128, N = 128, K = 32, A in tmem
+//   P3  (Q~ S_0)^T += W^T Bm^T  -> Y^T                 M = 128, N = 32, K = 32, A in tmem
+// Shared-memory operands are K-major core matrices (8 rows x 16 bytes). The
+// FMA pipe keeps the element-wise work, the triangular solve (I + A) W = R
+// (one value column per thread) and the scaling of S by g_C.
 //
 // One CTA (256 threads, 8 warps) per SM, persistent over (slot, value head)
 // items; it owns all 512 tensor-memory columns:
 //   [0, 128) S^T fp32 | [128, 256) S^T head | [256, 384) S^T rest |
-//   [384, 448) P1 result | [448, 480) W^T head | [480, 512) W^T rest.
+//   [384, 416) (K~ S_0)^T | [416, 448) (Q~ S_0)^T, then Y^T |
+//   [448, 480) P0 result, then W^T head | [480, 512) W^T rest.
 // Warps w and w + 4 share tensor-memory lanes 32 (w % 4) ..: the first four
-// warps solve for W, the last four scale the state by g_C, and both halves
-// split the column ranges of the loads and stores.
+// warps solve for W while the last four scale the state by g_C.
 #include "async.cuh"
 #include "device.cuh"
 #include "internal.h"
@@ -43,33 +43,50 @@ namespace stepq {
 namespace pf {
 
 constexpr int C = 32;                                  // tokens per chunk
-constexpr uint32_t kColS = 0, kColSh = 128, kColSl = 256, kColX = 384, kColWh = 448, kColWl = 480;
+constexpr uint32_t kColS = 0, kColSh = 128, kColSl = 256, kColX = 384, kColY = 416, kColP0 = 448,
+                   kColWh = 448, kColWl = 480;
 constexpr uint32_t kCols = 512;
-constexpr uint32_t kIdesc1 = tc::idesc_tf32(128, 64);
-constexpr uint32_t kIdesc2 = tc::idesc_tf32(128, 128);
+constexpr uint32_t kIdescP0 = tc::idesc_tf32(128, 32);
+constexpr uint32_t kIdescP1 = tc::idesc_tf32(128, 64);
+constexpr uint32_t kIdescP2 = tc::idesc_tf32(128, 128);
+constexpr uint32_t kIdescP3 = tc::idesc_tf32(128, 32);
 
-// shared memory (bytes); the MMA operands first, 1024-byte aligned
-constexpr int kOffB1h = 0;                             // [K~ ; Q~] head: 64 rows x K 128 (32 KB)
-constexpr int kOffB1l = kOffB1h + 32768;               // rest
-constexpr int kOffB2h = kOffB1l + 32768;               // K_bar^T head: 128 rows (i) x K 32 (t) (16 KB)
-constexpr int kOffB2l = kOffB2h + 16384;
-constexpr int kOffKt = kOffB2l + 16384;                // float [C][128] G K
-constexpr int kOffKh = kOffKt + C * 128 * 4;           // float [C][128] G^-1 K
-constexpr int kOffQt = kOffKh + C * 128 * 4;           // float [C][128] G Q
-constexpr int kOffV = kOffQt + C * 128 * 4;            // float [C][128] V
+// Shared-memory operands: K-major core matrices of 8 rows x 4 fp32 (128 B),
+// the core matrices of one row group 144 B apart along K (16 B of padding each,
+// so that a warp storing 32 consecutive K elements of one row hits 32 banks),
+// row groups kSbo128 / kSbo32 apart for K = 128 / 32.
+constexpr int kLbo = 144;
+constexpr int kSbo128 = 32 * kLbo;                     // 4608
+constexpr int kSbo32 = 8 * kLbo;                       // 1152
+// P0 reads 128 rows of A from B1: rows 64..127 fall on B1l and B3 (valid
+// memory; their results are unused).
+constexpr int kOffB1h = 0;                             // [K~ ; Q~] head: 64 rows x K 128
+constexpr int kOffB1l = kOffB1h + 8 * kSbo128;         // rest
+constexpr int kOffB3h = kOffB1l + 8 * kSbo128;         // K^ head: 32 rows (s) x K 128
+constexpr int kOffB3l = kOffB3h + 4 * kSbo128;
+constexpr int kOffB2h = kOffB3l + 4 * kSbo128;         // K_bar^T head: 128 rows (i) x K 32 (t)
+constexpr int kOffB2l = kOffB2h + 16 * kSbo32;
+constexpr int kOffB4h = kOffB2l + 16 * kSbo32;         // Bm head: 32 rows (t) x K 32 (s)
+constexpr int kOffB4l = kOffB4h + 4 * kSbo32;
+constexpr int kOffV = kOffB4l + 4 * kSbo32;            // float [C][128] V
 constexpr int kOffG = kOffV + C * 128 * 4;             // float [C][128] cumulative gates
-constexpr int kOffW = kOffG + C * 128 * 4;             // float [C][128] W
-constexpr int kOffA = kOffW + C * 128 * 4;             // float [C][C] A (strict lower)
-constexpr int kOffB = kOffA + C * C * 4;               // float [C][C] Q~ K^T (lower, with diagonal)
-constexpr int kOffBeta = kOffB + C * C * 4;            // float [C]
+constexpr int kOffA = kOffG + C * 128 * 4;             // float [C][C] A (strict lower)
+constexpr int kOffBeta = kOffA + C * C * 4;            // float [C]
 constexpr int kOffBar = kOffBeta + C * 4;              // uint64 mbarrier
 constexpr int kOffTmem = kOffBar + 8;                  // u32 tensor-memory base
 constexpr int kSmem = kOffTmem + 8;
+static_assert(kOffB1l + 16 * kSbo128 <= kSmem, "P0's unused A rows must stay inside shared memory");
 
-// Element (row r, k) of a K-major operand stored as core matrices of 8 rows x
-// 4 fp32: the matrix (r / 8, k / 4) sits at (r / 8) * sbo + (k / 4) * 128.
+// Byte offset of element (row r, k) of a K-major operand with row groups `sbo` apart.
 __device__ __forceinline__ int core_off(int r, int k, int sbo) {
-    return (r >> 3) * sbo + (k >> 2) * 128 + (r & 7) * 16 + (k & 3) * 4;
+    return (r >> 3) * sbo + (k >> 2) * kLbo + (r & 7) * 16 + (k & 3) * 4;
+}
+
+__device__ __forceinline__ void put_split(uint8_t *hi_base, uint8_t *lo_base, int off, float x) {
+    float hi, lo;
+    tc::split_tf32(x, hi, lo);
+    *(float *)(hi_base + off) = hi;
+    *(float *)(lo_base + off) = lo;
 }
 
 struct Args {
@@ -82,9 +99,9 @@ struct Args {
 __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
     extern __shared__ __align__(1024) uint8_t smem[];
     uint8_t *B1h = smem + kOffB1h, *B1l = smem + kOffB1l, *B2h = smem + kOffB2h, *B2l = smem + kOffB2l;
-    float *Kt = (float *)(smem + kOffKt), *Kh = (float *)(smem + kOffKh), *Qt = (float *)(smem + kOffQt);
-    float *V = (float *)(smem + kOffV), *G = (float *)(smem + kOffG), *Wm = (float *)(smem + kOffW);
-    float *A = (float *)(smem + kOffA), *Bm = (float *)(smem + kOffB), *bet = (float *)(smem + kOffBeta);
+    uint8_t *B3h = smem + kOffB3h, *B3l = smem + kOffB3l, *B4h = smem + kOffB4h, *B4l = smem + kOffB4l;
+    float *V = (float *)(smem + kOffV), *G = (float *)(smem + kOffG), *A = (float *)(smem + kOffA);
+    float *bet = (float *)(smem + kOffBeta);
     uint64_t *bar = (uint64_t *)(smem + kOffBar);
     uint32_t *tbase = (uint32_t *)(smem + kOffTmem);
     const int tid = threadIdx.x, w = tid >> 5, l = tid & 31;
@@ -106,19 +123,27 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
     uint32_t parity = 0;
     bool alive = true;
     const int grp = a.Hv / a.Hk;
+    // a CTA-wide bounded wait on the commit barrier; false if any thread gave up
+    const auto wait_mma = [&]() {
+        const bool ok = mbar_wait(bar, parity, pipe::kWaitCycles);
+        parity ^= 1u;
+        const bool stalled = __syncthreads_or(!ok);
+        tc::fence_after();
+        return !stalled;
+    };
     for (int item = blockIdx.x; alive && item < a.items; item += gridDim.x) {
         const int b = item / a.Hv, h = item - b * a.Hv, hk = h / grp;
         float *Sg = a.states + (size_t)item * kN;
         // S^T into tensor memory: this thread's lane j, the 64 key rows of its half.
         for (int c = 0; c < 2; c++) {
             const int i0 = 64 * half + 32 * c;
-            float s[32], hi[32], lo[32];
+            float sv[32], hi[32], lo[32];
 #pragma unroll
             for (int e = 0; e < 32; e++) {
-                s[e] = Sg[(size_t)(i0 + e) * 128 + j];
-                tc::split_tf32(s[e], hi[e], lo[e]);
+                sv[e] = Sg[(size_t)(i0 + e) * 128 + j];
+                tc::split_tf32(sv[e], hi[e], lo[e]);
             }
-            tc::st32(tl + kColS + i0, s);
+            tc::st32(tl + kColS + i0, sv);
             tc::st32(tl + kColSh + i0, hi);
             tc::st32(tl + kColSl + i0, lo);
         }
@@ -127,28 +152,9 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
             const int n = min(C, a.T - t0);               // tokens in this chunk (ragged tail)
             tc::fence_before();
             __syncthreads();                              // the previous chunk is done with every buffer
-            // Chunk operands; missing tokens of the tail are the identity step
-            // (gate 1, beta 0, zero k, q, v).
-#pragma unroll
-            for (int e = tid; e < C * 32; e += kThreads) {
-                const int t = e >> 5, c4 = e & 31;
-                float4 kq = make_float4(0.f, 0.f, 0.f, 0.f), qq = kq, vv = kq;
-                if (t < n) {
-                    const size_t tok = (size_t)b * a.T + t0 + t;
-                    kq = ((const float4 *)(a.k + (tok * a.Hk + hk) * 128))[c4];
-                    qq = ((const float4 *)(a.q + (tok * a.Hk + hk) * 128))[c4];
-                    vv = ((const float4 *)(a.v + (tok * a.Hv + h) * 128))[c4];
-                }
-                ((float4 *)Kt)[e] = kq;                   // raw k until the gates are known
-                ((float4 *)Qt)[e] = qq;
-                ((float4 *)V)[e] = vv;
-            }
-            if (tid < C) {
-                const size_t tok = (size_t)b * a.T + t0 + tid;
-                bet[tid] = tid < n ? a.beta[tok * a.Hv + h] : 0.f;
-            }
-            // Cumulative gates g_t per key channel: the chunk's 32 gates are loaded
-            // at once (independent loads), then multiplied in token order.
+            // Cumulative gates g_t per key channel (the chunk's 32 gates loaded at
+            // once, then multiplied in token order) and beta. Missing tokens of
+            // the tail are the identity step (gate 1, beta 0, zero k, q, v).
             if (tid < 128) {
                 float d[C];
 #pragma unroll
@@ -164,75 +170,79 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
                     g = fmaxf(g * d[t], 1e-30f);          // keeps K / g finite
                     G[t * 128 + tid] = g;
                 }
+            } else if (tid < 128 + C) {
+                const int t = tid - 128;
+                bet[t] = t < n ? a.beta[((size_t)b * a.T + t0 + t) * a.Hv + h] : 0.f;
             }
             __syncthreads();
-            // K~ = G K, K^ = K / G, Q~ = G Q (fp32), and the split MMA operands
-            // [K~ ; Q~] and K_bar^T with K_bar = K g_C / g.
-            for (int e = tid; e < C * 128; e += kThreads) {
-                const int t = e >> 7, i = e & 127;
-                const float g = G[e], kv = Kt[e];
-                const float kt = g * kv, qt = Qt[e] * g, kb = kv * (G[(C - 1) * 128 + i] / g);
-                Kt[e] = kt;
-                Kh[e] = kv / g;
-                Qt[e] = qt;
-                float hi, lo;
-                tc::split_tf32(kt, hi, lo);
-                *(float *)(B1h + core_off(t, i, 4096)) = hi;
-                *(float *)(B1l + core_off(t, i, 4096)) = lo;
-                tc::split_tf32(qt, hi, lo);
-                *(float *)(B1h + core_off(C + t, i, 4096)) = hi;
-                *(float *)(B1l + core_off(C + t, i, 4096)) = lo;
-                tc::split_tf32(kb, hi, lo);
-                *(float *)(B2h + core_off(i, t, 1024)) = hi;
-                *(float *)(B2l + core_off(i, t, 1024)) = lo;
+            // Element-wise: V, and the split operands [K~ ; Q~], K^ and K_bar^T.
+            // Thread: key channel i, tokens tb, tb + 2, ..., tb + 30.
+            {
+                const int i = tid & 127, tb = tid >> 7;
+                float kv[C / 2], qv[C / 2], vv[C / 2];
+#pragma unroll
+                for (int u = 0; u < C / 2; u++) {
+                    const int t = tb + 2 * u;
+                    kv[u] = qv[u] = vv[u] = 0.f;
+                    if (t < n) {
+                        const size_t tok = (size_t)b * a.T + t0 + t;
+                        kv[u] = a.k[(tok * a.Hk + hk) * 128 + i];
+                        qv[u] = a.q[(tok * a.Hk + hk) * 128 + i];
+                        vv[u] = a.v[(tok * a.Hv + h) * 128 + i];
+                    }
+                }
+                const float gC = G[(C - 1) * 128 + i];
+#pragma unroll
+                for (int u = 0; u < C / 2; u++) {
+                    const int t = tb + 2 * u;
+                    const float g = G[t * 128 + i], rg = 1.0f / g;
+                    V[t * 128 + i] = vv[u];
+                    put_split(B1h, B1l, core_off(t, i, kSbo128), g * kv[u]);        // K~
+                    put_split(B1h, B1l, core_off(C + t, i, kSbo128), g * qv[u]);    // Q~
+                    put_split(B3h, B3l, core_off(t, i, kSbo128), kv[u] * rg);       // K^
+                    put_split(B2h, B2l, core_off(i, t, kSbo32), kv[u] * (gC * rg)); // K_bar^T
+                }
             }
             fence_async_smem();                           // operands visible to the tensor cores
             __syncthreads();
-            // P1: [K~ S_0 ; Q~ S_0]^T into columns [384, 448), 16 steps of K = 8.
+            // P0: [K~ ; Q~] K^T into columns [448, 480); P1: [K~ S_0 ; Q~ S_0]^T into [384, 448).
             if (tid == 0) {
                 tc::fence_after();
 #pragma unroll 1
                 for (int s = 0; s < 16; s++) {
-                    const uint64_t bh = tc::sdesc(B1h + 256 * s, 128, 4096);
-                    const uint64_t bl = tc::sdesc(B1l + 256 * s, 128, 4096);
-                    tc::mma_tf32_ts(tm + kColX, tm + kColSh + 8 * s, bh, kIdesc1, s > 0 ? 1u : 0u);
-                    tc::mma_tf32_ts(tm + kColX, tm + kColSh + 8 * s, bl, kIdesc1, 1u);
-                    tc::mma_tf32_ts(tm + kColX, tm + kColSl + 8 * s, bh, kIdesc1, 1u);
+                    const uint64_t ah = tc::sdesc(B1h + 2 * kLbo * s, kLbo, kSbo128), al = tc::sdesc(B1l + 2 * kLbo * s, kLbo, kSbo128);
+                    const uint64_t kh = tc::sdesc(B3h + 2 * kLbo * s, kLbo, kSbo128), kl = tc::sdesc(B3l + 2 * kLbo * s, kLbo, kSbo128);
+                    const uint32_t acc = s > 0 ? 1u : 0u;
+                    tc::mma_tf32_ss(tm + kColP0, ah, kh, kIdescP0, acc);
+                    tc::mma_tf32_ss(tm + kColP0, ah, kl, kIdescP0, 1u);
+                    tc::mma_tf32_ss(tm + kColP0, al, kh, kIdescP0, 1u);
+                    tc::mma_tf32_ts(tm + kColX, tm + kColSh + 8 * s, ah, kIdescP1, acc);
+                    tc::mma_tf32_ts(tm + kColX, tm + kColSh + 8 * s, al, kIdescP1, 1u);
+                    tc::mma_tf32_ts(tm + kColX, tm + kColSl + 8 * s, ah, kIdescP1, 1u);
                 }
                 tc::commit(bar);
             }
-            __syncwarp();                                 // warp 0 converged again
-            // Meanwhile on the FMA pipe: A = strict lower of diag(beta) K~ K^T,
-            // Bm = lower (with diagonal) of Q~ K^T.
-            {
-                const int t = tid >> 3, s0 = (tid & 7) * 4;
-                float ac[4] = {0.f, 0.f, 0.f, 0.f}, bc[4] = {0.f, 0.f, 0.f, 0.f};
-                for (int i4 = 0; i4 < 32; i4++) {
-                    const float4 kt = ((const float4 *)(Kt + t * 128))[i4];
-                    const float4 qt = ((const float4 *)(Qt + t * 128))[i4];
+            __syncwarp();
+            if (!wait_mma()) {
+                alive = false;
+                break;
+            }
+            // A = strict lower of diag(beta) K~ K^T (row t = lane t) and Bm =
+            // lower (with diagonal) of Q~ K^T (row t = lane 32 + t), Bm split as an operand.
+            if (w < 2) {
+                float d[32];
+                tc::ld32(tl + kColP0, d);
+                if (w == 0) {
+                    const float bt = bet[l];
 #pragma unroll
-                    for (int c = 0; c < 4; c++) {
-                        const float4 kh = ((const float4 *)(Kh + (s0 + c) * 128))[i4];
-                        ac[c] += kt.x * kh.x + kt.y * kh.y + kt.z * kh.z + kt.w * kh.w;
-                        bc[c] += qt.x * kh.x + qt.y * kh.y + qt.z * kh.z + qt.w * kh.w;
-                    }
-                }
+                    for (int s = 0; s < C; s++) A[l * C + s] = s < l ? bt * d[s] : 0.f;
+                } else {
 #pragma unroll
-                for (int c = 0; c < 4; c++) {
-                    const int s = s0 + c;
-                    A[t * C + s] = s < t ? bet[t] * ac[c] : 0.f;
-                    Bm[t * C + s] = s <= t ? bc[c] : 0.f;
+                    for (int s = 0; s < C; s++) put_split(B4h, B4l, core_off(l, s, kSbo32), s <= l ? d[s] : 0.f);
+                    fence_async_smem();
                 }
             }
-            {
-                const bool ok = mbar_wait(bar, parity, pipe::kWaitCycles);
-                parity ^= 1u;
-                if (__syncthreads_or(!ok)) {              // A, Bm visible as well
-                    alive = false;
-                    break;
-                }
-            }
-            tc::fence_after();
+            __syncthreads();                              // A visible; P0's columns free for W
             if (half == 0) {
                 // W = (I + A)^-1 diag(beta) (V - K~ S_0), value column j.
                 float x[32], wv[32];
@@ -241,73 +251,72 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
                 for (int t = 0; t < C; t++) {
                     float acc = bet[t] * (V[t * 128 + j] - x[t]);
 #pragma unroll
-                    for (int s = 0; s < t; s++) acc -= A[t * C + s] * wv[s];
+                    for (int s4 = 0; 4 * s4 < t; s4++) {           // A row t, four at a time
+                        const float4 a4 = ((const float4 *)(A + t * C))[s4];
+                        const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+                        for (int e = 0; e < 4; e++)
+                            if (4 * s4 + e < t) acc -= av[e] * wv[4 * s4 + e];
+                    }
                     wv[t] = acc;
                 }
                 float hi[32], lo[32];
 #pragma unroll
-                for (int t = 0; t < C; t++) {
-                    Wm[t * 128 + j] = wv[t];
-                    tc::split_tf32(wv[t], hi[t], lo[t]);
-                }
+                for (int t = 0; t < C; t++) tc::split_tf32(wv[t], hi[t], lo[t]);
                 tc::st32(tl + kColWh, hi);
                 tc::st32(tl + kColWl, lo);
             } else {
                 // S^T <- S^T diag(g_C): key row i scaled by its cumulative gate.
 #pragma unroll 1
                 for (int c = 0; c < 4; c++) {
-                    float s[32];
-                    tc::ld32(tl + kColS + 32 * c, s);
+                    float sv[32];
+                    tc::ld32(tl + kColS + 32 * c, sv);
 #pragma unroll
-                    for (int e = 0; e < 32; e++) s[e] *= G[(C - 1) * 128 + 32 * c + e];
-                    tc::st32(tl + kColS + 32 * c, s);
+                    for (int e = 0; e < 32; e++) sv[e] *= G[(C - 1) * 128 + 32 * c + e];
+                    tc::st32(tl + kColS + 32 * c, sv);
                 }
             }
             tc::wait_st();
             tc::fence_before();
             __syncthreads();
-            // P2: S^T += W^T K_bar, 4 steps of K = 8.
+            // P2: S^T += W^T K_bar; P3: Y^T = (Q~ S_0)^T + W^T Bm^T.
             if (tid == 0) {
                 tc::fence_after();
 #pragma unroll 1
                 for (int s = 0; s < 4; s++) {
-                    const uint64_t bh = tc::sdesc(B2h + 256 * s, 128, 1024);
-                    const uint64_t bl = tc::sdesc(B2l + 256 * s, 128, 1024);
-                    tc::mma_tf32_ts(tm + kColS, tm + kColWh + 8 * s, bh, kIdesc2, 1u);
-                    tc::mma_tf32_ts(tm + kColS, tm + kColWh + 8 * s, bl, kIdesc2, 1u);
-                    tc::mma_tf32_ts(tm + kColS, tm + kColWl + 8 * s, bh, kIdesc2, 1u);
+                    const uint64_t bh = tc::sdesc(B2h + 2 * kLbo * s, kLbo, kSbo32), bl = tc::sdesc(B2l + 2 * kLbo * s, kLbo, kSbo32);
+                    const uint64_t mh = tc::sdesc(B4h + 2 * kLbo * s, kLbo, kSbo32), ml = tc::sdesc(B4l + 2 * kLbo * s, kLbo, kSbo32);
+                    tc::mma_tf32_ts(tm + kColS, tm + kColWh + 8 * s, bh, kIdescP2, 1u);
+                    tc::mma_tf32_ts(tm + kColS, tm + kColWh + 8 * s, bl, kIdescP2, 1u);
+                    tc::mma_tf32_ts(tm + kColS, tm + kColWl + 8 * s, bh, kIdescP2, 1u);
+                    tc::mma_tf32_ts(tm + kColY, tm + kColWh + 8 * s, mh, kIdescP3, 1u);
+                    tc::mma_tf32_ts(tm + kColY, tm + kColWh + 8 * s, ml, kIdescP3, 1u);
+                    tc::mma_tf32_ts(tm + kColY, tm + kColWl + 8 * s, mh, kIdescP3, 1u);
                 }
                 tc::commit(bar);
             }
-            __syncwarp();                                 // warp 0 converged before tcgen05.ld
-            // Meanwhile: Y = Q~ S_0 + Bm W, tokens 16 half .. 16 half + 15 of column j.
+            __syncwarp();
+            if (!wait_mma()) {
+                alive = false;
+                break;
+            }
+            // Outputs: tokens 16 half .. 16 half + 15 of column j.
             {
-                float yo[16];
-                tc::ld16(tl + kColX + 32 + 16 * half, yo);
-#pragma unroll 4
-                for (int u = 0; u < 16; u++) {
-                    const int t = 16 * half + u;
-                    float acc = yo[u];
-                    for (int s = 0; s <= t; s++) acc += Bm[t * C + s] * Wm[s * 128 + j];
-                    if (t < n) a.y[(((size_t)b * a.T + t0 + t) * a.Hv + h) * 128 + j] = acc;
+                float yv[16];
+                tc::ld16(tl + kColY + 16 * half, yv);
+#pragma unroll
+                for (int e = 0; e < 16; e++) {
+                    const int t = 16 * half + e;
+                    if (t < n) a.y[(((size_t)b * a.T + t0 + t) * a.Hv + h) * 128 + j] = yv[e];
                 }
             }
-            {
-                const bool ok = mbar_wait(bar, parity, pipe::kWaitCycles);
-                parity ^= 1u;
-                if (__syncthreads_or(!ok)) {
-                    alive = false;
-                    break;
-                }
-            }
-            tc::fence_after();
             // Heads and rests of the new state for the next chunk's P1.
             for (int c = 0; c < 2; c++) {
                 const int i0 = 64 * half + 32 * c;
-                float s[32], hi[32], lo[32];
-                tc::ld32(tl + kColS + i0, s);
+                float sv[32], hi[32], lo[32];
+                tc::ld32(tl + kColS + i0, sv);
 #pragma unroll
-                for (int e = 0; e < 32; e++) tc::split_tf32(s[e], hi[e], lo[e]);
+                for (int e = 0; e < 32; e++) tc::split_tf32(sv[e], hi[e], lo[e]);
                 tc::st32(tl + kColSh + i0, hi);
                 tc::st32(tl + kColSl + i0, lo);
             }
@@ -317,10 +326,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
         // The boundary state back to global memory.
         for (int c = 0; c < 2; c++) {
             const int i0 = 64 * half + 32 * c;
-            float s[32];
-            tc::ld32(tl + kColS + i0, s);
+            float sv[32];
+            tc::ld32(tl + kColS + i0, sv);
 #pragma unroll
-            for (int e = 0; e < 32; e++) Sg[(size_t)(i0 + e) * 128 + j] = s[e];
+            for (int e = 0; e < 32; e++) Sg[(size_t)(i0 + e) * 128 + j] = sv[e];
         }
     }
     if (!alive && tid == 0) {
