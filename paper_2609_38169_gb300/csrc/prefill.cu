@@ -131,8 +131,43 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
         tc::fence_after();
         return !stalled;
     };
+    // This thread's share of a chunk's operands, loaded one chunk ahead (their
+    // global-memory latency overlaps the previous chunk's tensor-core work):
+    // key channel ci at tokens tb, tb + 2, ..., tb + 30 of k, q, v; threads
+    // 0..127 the chunk's gates of channel ci, threads 128..159 one beta each.
+    // Missing tokens of a ragged tail are the identity step (gate 1, beta 0,
+    // zero k, q, v).
+    const int ci = tid & 127, tb = tid >> 7;
+    float kv[C / 2], qv[C / 2], vv[C / 2], dg[C], bt = 0.f;
+    const auto fetch = [&](int it, int c0) {
+        const int fb = it / a.Hv, fh = it - fb * a.Hv, fhk = fh / grp, fn = min(C, a.T - c0);
+#pragma unroll
+        for (int u = 0; u < C / 2; u++) {
+            const int t = tb + 2 * u;
+            kv[u] = qv[u] = vv[u] = 0.f;
+            if (t < fn) {
+                const size_t tok = (size_t)fb * a.T + c0 + t;
+                kv[u] = a.k[(tok * a.Hk + fhk) * 128 + ci];
+                qv[u] = a.q[(tok * a.Hk + fhk) * 128 + ci];
+                vv[u] = a.v[(tok * a.Hv + fh) * 128 + ci];
+            }
+        }
+        if (tid < 128) {
+#pragma unroll
+            for (int t = 0; t < C; t++) {
+                const size_t tok = (size_t)fb * a.T + c0 + t;
+                float dv = 1.f;
+                if (t < fn) dv = a.gate_per_row ? a.gate[(tok * a.Hv + fh) * 128 + ci] : a.gate[tok * a.Hv + fh];
+                dg[t] = dv;
+            }
+        } else if (tid < 128 + C) {
+            const int t = tid - 128;
+            bt = t < fn ? a.beta[((size_t)fb * a.T + c0 + t) * a.Hv + fh] : 0.f;
+        }
+    };
+    if ((int)blockIdx.x < a.items) fetch(blockIdx.x, 0);
     for (int item = blockIdx.x; alive && item < a.items; item += gridDim.x) {
-        const int b = item / a.Hv, h = item - b * a.Hv, hk = h / grp;
+        const int b = item / a.Hv, h = item - b * a.Hv;
         float *Sg = a.states + (size_t)item * kN;
         // S^T into tensor memory: this thread's lane j, the 64 key rows of its half.
         for (int c = 0; c < 2; c++) {
@@ -152,45 +187,21 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
             const int n = min(C, a.T - t0);               // tokens in this chunk (ragged tail)
             tc::fence_before();
             __syncthreads();                              // the previous chunk is done with every buffer
-            // Cumulative gates g_t per key channel (the chunk's 32 gates loaded at
-            // once, then multiplied in token order) and beta. Missing tokens of
-            // the tail are the identity step (gate 1, beta 0, zero k, q, v).
+            // Cumulative gates g_t per key channel (multiplied in token order) and beta.
             if (tid < 128) {
-                float d[C];
-#pragma unroll
-                for (int t = 0; t < C; t++) {
-                    const size_t tok = (size_t)b * a.T + t0 + t;
-                    float dv = 1.f;
-                    if (t < n) dv = a.gate_per_row ? a.gate[(tok * a.Hv + h) * 128 + tid] : a.gate[tok * a.Hv + h];
-                    d[t] = dv;
-                }
                 float g = 1.f;
 #pragma unroll
                 for (int t = 0; t < C; t++) {
-                    g = fmaxf(g * d[t], 1e-30f);          // keeps K / g finite
+                    g = fmaxf(g * dg[t], 1e-30f);         // keeps K / g finite
                     G[t * 128 + tid] = g;
                 }
             } else if (tid < 128 + C) {
-                const int t = tid - 128;
-                bet[t] = t < n ? a.beta[((size_t)b * a.T + t0 + t) * a.Hv + h] : 0.f;
+                bet[tid - 128] = bt;
             }
             __syncthreads();
             // Element-wise: V, and the split operands [K~ ; Q~], K^ and K_bar^T.
-            // Thread: key channel i, tokens tb, tb + 2, ..., tb + 30.
             {
-                const int i = tid & 127, tb = tid >> 7;
-                float kv[C / 2], qv[C / 2], vv[C / 2];
-#pragma unroll
-                for (int u = 0; u < C / 2; u++) {
-                    const int t = tb + 2 * u;
-                    kv[u] = qv[u] = vv[u] = 0.f;
-                    if (t < n) {
-                        const size_t tok = (size_t)b * a.T + t0 + t;
-                        kv[u] = a.k[(tok * a.Hk + hk) * 128 + i];
-                        qv[u] = a.q[(tok * a.Hk + hk) * 128 + i];
-                        vv[u] = a.v[(tok * a.Hv + h) * 128 + i];
-                    }
-                }
+                const int i = ci;
                 const float gC = G[(C - 1) * 128 + i];
 #pragma unroll
                 for (int u = 0; u < C / 2; u++) {
@@ -296,6 +307,14 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
                 tc::commit(bar);
             }
             __syncwarp();
+            {   // the next chunk's operands: this item's next chunk or the next item's first
+                int ni = item, nt = t0 + C;
+                if (nt >= a.T) {
+                    ni += gridDim.x;
+                    nt = 0;
+                }
+                if (ni < a.items) fetch(ni, nt);
+            }
             if (!wait_mma()) {
                 alive = false;
                 break;
