@@ -206,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
 #pragma unroll
                 for (int u = 0; u < C / 2; u++) {
                     const int t = tb + 2 * u;
-                    const float g = G[t * 128 + i], rg = 1.0f / g;
+                    const float g = G[t * 128 + i], rg = __fdividef(1.0f, g);   // within 2 ulp
                     V[t * 128 + i] = vv[u];
                     put_split(B1h, B1l, core_off(t, i, kSbo128), g * kv[u]);        // K~
                     put_split(B1h, B1l, core_off(C + t, i, kSbo128), g * qv[u]);    // Q~
