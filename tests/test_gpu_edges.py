@@ -1,0 +1,101 @@
+"""Edge cases of the decode path against the oracle (App. C.3 steps 1-7):
+degenerate states and the largest head count a launch accepts.
+
+States: an all-zero state (every scale at its FP16 floor, codes 0), states
+scaled by 1e9 (the clip-free column start exceeds the FP16 range, so the
+codes take the clamped path), states scaled by 1e-12 (row factors at the
+FP16 floor) and a state of tiny values with a few large outliers. Each runs
+two teacher-forced decode steps under the parity rules of gpu_helpers.
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2609_38169_gb300 import api as A, workloads as W
+
+from gpu_helpers import Tally, compare_pools, compare_y, plans, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    import torch as T
+    if not T.cuda.is_available():
+        pytest.skip("no CUDA device")
+    return T
+
+
+def _degenerate_states(wl, B=4):
+    base = W.random_states(wl, B * wl.hv, seed=21).reshape(B, wl.hv, 128, 128).astype(np.float64)
+    S = np.zeros_like(base)                                   # slot 0: zero state
+    S[1] = base[1] * 1e9                                      # slot 1: huge
+    S[2] = base[2] * 1e-12                                    # slot 2: tiny
+    S[3] = base[3] * 1e-6                                     # slot 3: tiny with outliers
+    rng = np.random.default_rng(5)
+    for h in range(wl.hv):
+        idx = rng.integers(0, 128, size=(3, 2))
+        S[3, h, idx[:, 0], idx[:, 1]] = rng.choice([-1.0, 1.0], 3) * 1e3
+    return S.astype(np.float32)
+
+
+def _teacher_forced(torch, wl, S, steps=2):
+    cfg, plan, oplan, _ = plans(wl)
+    mp = W.model_params(wl)
+    B = S.shape[0]
+    slots = np.arange(B, dtype=np.int32)[::-1].copy()
+    pool_o = np.zeros(wl.pool_slots * oplan.slot_stride, np.uint8)
+    O.pool_encode(oplan, pool_o, 0, slots, S)
+    pool_d = A.alloc_pool(plan, wl.pool_slots)
+    (slots_d, S_d) = to_dev(slots, S)
+    A.stepq_quantize_pool(plan, 0, S_d, slots_d, pool_d)
+    t = Tally()
+    compare_pools(t, pool_d.cpu().numpy(), pool_o, oplan, 0, slots)
+    for step in range(steps):
+        inp = W.step_inputs(wl, mp, W.STREAM_DECODE, step, 0, batch=B)
+        pool_d.copy_(torch.from_numpy(pool_o))
+        q, k, v, beta, gate = to_dev(inp.q, inp.k, inp.v, inp.beta, inp.gate)
+        y_d = torch.empty((B, wl.hv, 128), dtype=torch.float32, device="cuda")
+        A.stepq_decode_step(plan, 0, pool_d, slots_d, q, k, v, beta, gate, y_d)
+        y_o = O.pool_step(oplan, pool_o, 0, slots, inp)
+        assert np.isfinite(y_d.cpu().numpy()).all()
+        compare_y(t, y_d.cpu().numpy(), y_o)
+        compare_pools(t, pool_d.cpu().numpy(), pool_o, oplan, 0, slots)
+    return t
+
+
+@pytest.mark.parametrize("name,kw", [("gqa", dict(n_pivots=3, pool_slots=4)),
+                                     ("channel", dict(pool_slots=4))])
+def test_degenerate_states(torch, name, kw):
+    wl = W.WORKLOADS[name].replace(**kw)
+    t = _teacher_forced(torch, wl, _degenerate_states(wl))
+    print(name, t.summary())
+    t.check()
+    assert A.stepq_device_error() == 0
+
+
+def test_largest_head_count(torch):
+    """256 value heads (64 key heads) per layer, the most one launch takes."""
+    wl = W.WORKLOADS["gqa"].replace(name="maxheads", hk=64, hv=256, batch=2, pool_slots=4, n_pivots=5)
+    S = W.random_states(wl, 2 * wl.hv, seed=9).reshape(2, wl.hv, 128, 128)
+    t = _teacher_forced(torch, wl, S)
+    print(t.summary())
+    t.check()
+    assert A.stepq_device_error() == 0
+
+
+def test_too_many_heads_is_refused(torch):
+    """More value heads than a launch supports: an error before any launch."""
+    wl = W.WORKLOADS["gqa"].replace(name="toomany", hk=64, hv=320, batch=1, pool_slots=1)
+    cfg, plan, oplan, _ = plans(wl, seqs=1, steps=4)
+    pool_d = A.alloc_pool(plan, 1)
+    before = pool_d.clone()
+    z = torch.zeros((1, wl.hk, 128), device="cuda")
+    zv = torch.zeros((1, wl.hv, 128), device="cuda")
+    beta = torch.zeros((1, wl.hv), device="cuda")
+    gate = torch.ones((1, wl.hv), device="cuda")
+    slots = torch.zeros(1, dtype=torch.int32, device="cuda")
+    with pytest.raises(A._lib.StepqError):
+        A.stepq_decode_step(plan, 0, pool_d, slots, z, z, zv, beta, gate, zv.clone())
+    assert torch.equal(pool_d, before)
+    assert A.stepq_device_error() == 0
