@@ -316,22 +316,46 @@ def main():
                 "avg_launch_us": avg_launch_s * 1e6}
 
     # ---- end to end through the public API with host buffers ----
+    # Every step copies each layer's inputs from pinned host memory and reads
+    # every layer's y back. The copies run on their own streams, one layer
+    # ahead of / behind the kernel that uses them (two device input buffers,
+    # ordered by events), so they overlap the decode kernels; the step ends
+    # when the last y has reached the host.
     h_in = []
     for layer in range(L):
         h_in.append([x.cpu().pin_memory() for x in inputs[0][layer]])
-    d_in = [[torch.empty_like(x) for x in inputs[0][layer]] for layer in range(L)]
+    d_in = [[torch.empty_like(x) for x in inputs[0][0]] for _ in range(2)]
     h_y = torch.empty((L, B, Hv, 128), dtype=torch.float32).pin_memory()
     h2d = sum(x.numel() * x.element_size() for row in h_in for x in row)
     d2h = h_y.numel() * 4
+    h2d_stream, d2h_stream = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    buf_free = [torch.cuda.Event() for _ in range(2)]
+    copied = [torch.cuda.Event() for _ in range(2)]
+    y_done = [torch.cuda.Event() for _ in range(L)]
+    y_read = [torch.cuda.Event() for _ in range(L)]
+    for e in buf_free + y_read:
+        e.record(stream)
 
     def step_e2e(s):
         for layer in range(L):
-            for dst, src in zip(d_in[layer], h_in[layer]):
-                dst.copy_(src, non_blocking=True)
-            q, k, v, beta, gate = d_in[layer]
+            nb = (s * L + layer) % 2
+            h2d_stream.wait_event(buf_free[nb])         # the kernel that last read this buffer
+            with torch.cuda.stream(h2d_stream):
+                for dst, src in zip(d_in[nb], h_in[layer]):
+                    dst.copy_(src, non_blocking=True)
+                copied[nb].record(h2d_stream)
+            stream.wait_event(copied[nb])
+            stream.wait_event(y_read[layer])            # last step's y of this layer is on the host
+            q, k, v, beta, gate = d_in[nb]
             P.stepq_decode_step(plan, layer, pool, slots, q, k, v, beta, gate, y[layer],
-                                pool_slots=wl.pool_slots)
-        h_y.copy_(y, non_blocking=True)
+                                pool_slots=wl.pool_slots, stream=stream)
+            buf_free[nb].record(stream)
+            y_done[layer].record(stream)
+            d2h_stream.wait_event(y_done[layer])
+            with torch.cuda.stream(d2h_stream):
+                h_y[layer].copy_(y[layer], non_blocking=True)
+                y_read[layer].record(d2h_stream)
+        stream.wait_event(y_read[L - 1])                # the step ends with y on the host
 
     e2e_steps = max(3, args.steps // 2)
     e2e_ms, _ = timed(step_e2e, e2e_steps, 2, name="stepq_e2e")
