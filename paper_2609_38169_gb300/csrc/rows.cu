@@ -210,6 +210,17 @@ __device__ __forceinline__ void load_pair(const T &t, const Smem &S, const uint8
     const uint4 inf = *(const uint4 *)&S.rInfo[t.row(2 * m)];
     const int b0 = (int)((inf.x >> 16) & 0xFFu), b1 = (int)((inf.z >> 16) & 0xFFu);
     const uint8_t *r0 = page + (inf.x & 0xFFFFu), *r1 = page + (inf.z & 0xFFFFu);
+    if (b0 != kPivot && b1 != kPivot) {                  // two integer rows: paired arithmetic
+        const uint32_t s0 = lane_segment(r0, b0, t.l), s1 = lane_segment(r1, b1, t.l);
+        const uint32_t k0 = (1u << b0) - 1u, k1 = (1u << b1) - 1u;
+        const uint64_t off = row_pair(S.rOff, t, m);
+#pragma unroll
+        for (int c = 0; c < 4; c++)
+            x[c] = fmul2(fadd2(u2pair(and_or(s0 >> (c * b0), k0, kMagicBits), and_or(s1 >> (c * b1), k1, kMagicBits)),
+                               off),
+                         cd[c]);
+        return;
+    }
     float v[2][4];
 #pragma unroll
     for (int h = 0; h < 2; h++) {
