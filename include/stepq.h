@@ -190,8 +190,7 @@ stepq_status stepq_prefill_fp32(const stepq_config *cfg, int B, int T, float *st
 /* The decode step split in two for a side stream (Sec. 4.4, App. F.1: after the
  * readout, scale fitting and packed writeback run on a separate CUDA stream
  * while later layers process the token; writeback completes before the next
- * recurrent step reads the state). Head-unit (scalar-gate) plans only;
- * row-unit plans return STEPQ_ERR_UNSUPPORTED.
+ * recurrent step reads the state). Head-unit and row-unit plans.
  *
  * stepq_decode_readout: App. C.3 steps 1-3 of stepq_decode_step: reconstruct,
  *   Delta update, readout. Writes y [B][Hv][128] and delta [B][Hv][128]

@@ -134,11 +134,13 @@ extern "C" stepq_status stepq_decode_readout(const stepq_plan *p, int layer, con
                                              float *delta, stepq_stream_t stream) {
     stepq_status st = check_plan_call(p, layer, false, pool, pool_slots, slots, B);
     if (st != STEPQ_OK) return st;
-    if (p->cfg.gate_kind == STEPQ_GATE_CHANNEL) return STEPQ_ERR_UNSUPPORTED;
     if (!v || !y || !delta) return STEPQ_ERR_ARG;
     if ((st = check_inputs(&p->cfg, q, k, v, beta, gate, y)) != STEPQ_OK) return st;
     if (!aligned(delta, 16)) return STEPQ_ERR_ALIGN;
     if (B == 0) return STEPQ_OK;
+    if (p->cfg.gate_kind == STEPQ_GATE_CHANNEL)
+        return launch_decode_rows_mode(p, layer, (uint8_t *)pool, pool_slots, slots, B, q, k, v, beta,
+                                       gate, y, delta, 1, (cudaStream_t)stream);
     return launch_decode_heads_mode(p, layer, (uint8_t *)pool, pool_slots, slots, B, q, k, v, beta,
                                     gate, y, delta, 1, (cudaStream_t)stream);
 }
@@ -150,11 +152,15 @@ extern "C" stepq_status stepq_decode_writeback(const stepq_plan *p, int layer, v
                                                stepq_stream_t stream) {
     stepq_status st = check_plan_call(p, layer, false, pool, pool_slots, slots, B);
     if (st != STEPQ_OK) return st;
-    if (p->cfg.gate_kind == STEPQ_GATE_CHANNEL) return STEPQ_ERR_UNSUPPORTED;
     if (!k || !beta || !gate || !delta) return STEPQ_ERR_ARG;
-    if (!aligned(k, 16) || !aligned(delta, 16) || !aligned(beta, 4) || !aligned(gate, 4))
+    if (!aligned(k, 16) || !aligned(delta, 16) || !aligned(beta, 4) ||
+        !aligned(gate, p->cfg.gate_kind == STEPQ_GATE_CHANNEL ? 16 : 4))
         return STEPQ_ERR_ALIGN;
     if (B == 0) return STEPQ_OK;
+    if (p->cfg.gate_kind == STEPQ_GATE_CHANNEL)
+        return launch_decode_rows_mode(p, layer, (uint8_t *)pool, pool_slots, slots, B, nullptr, k,
+                                       nullptr, beta, gate, nullptr, (float *)delta, 2,
+                                       (cudaStream_t)stream);
     return launch_decode_heads_mode(p, layer, (uint8_t *)pool, pool_slots, slots, B, nullptr, k,
                                     nullptr, beta, gate, nullptr, (float *)delta, 2,
                                     (cudaStream_t)stream);

@@ -104,6 +104,10 @@ stepq_status launch_decode_rows(const stepq_plan *p, int layer, uint8_t *pool, i
                                 const int32_t *slots, int B, const float *q, const float *k,
                                 const float *v, const float *beta, const float *gate, float *y,
                                 cudaStream_t s);
+stepq_status launch_decode_rows_mode(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
+                                     const int32_t *slots, int B, const float *q, const float *k,
+                                     const float *v, const float *beta, const float *gate, float *y,
+                                     float *delta, int mode, cudaStream_t s);
 // heads.cu (head units, band-major pages)
 stepq_status launch_decode_heads(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
                                  const int32_t *slots, int B, const float *q, const float *k,

@@ -181,25 +181,35 @@ struct DecodeArgs {
     LayerTables tab;
     const float *q, *k, *v, *beta, *gate;
     float *y;
+    float *delta;              // readout: delta_j out; writeback: delta_j in
     unsigned int *err;
     int n_stages;
     uint32_t page_region, stage_bytes;
     int fit_iters;
 };
 
+// Kernel modes as for the head-unit kernel: the fused step, the readout (y and
+// delta, page untouched) and the writeback (delta in; refit and pack).
+enum : int { kFused = 0, kReadout = 1, kWriteback = 2 };
+
+template <int MODE>
 __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s) {
     uint64_t *bar = &S.bars[s];
     Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
     const uint32_t nb = S.hbytes[h];
     const int hk = S.hkey[h];
-    mbar_arrive_tx(bar, nb + kVecBytes);
+    constexpr uint32_t vec = MODE == kFused ? kVecBytes : kVecBytes - (MODE == kReadout ? 1024 : 512);
+    mbar_arrive_tx(bar, nb + vec);
     bulk_load(st.page, a.pool + (uint64_t)slot * a.stride + S.hoff[h], nb, bar);
-    bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
+    if (MODE != kWriteback) bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
     bulk_load(st.k, a.k + ((size_t)b * a.Hk + hk) * 128, 512, bar);
-    bulk_load(st.v, a.v + ((size_t)b * a.Hv + h) * 128, 512, bar);
+    if (MODE != kWriteback) bulk_load(st.v, a.v + ((size_t)b * a.Hv + h) * 128, 512, bar);
+    else bulk_load(st.v, a.delta + ((size_t)b * a.Hv + h) * 128, 512, bar);
     bulk_load(st.gate, a.gate + ((size_t)b * a.Hv + h) * 128, 512, bar);
-    bulk_load(st.w2, a.tab.w2 + (size_t)h * 128, 512, bar);
-    bulk_load(st.wis, a.tab.wis + (size_t)h * 128, 512, bar);
+    if (MODE != kReadout) {
+        bulk_load(st.w2, a.tab.w2 + (size_t)h * 128, 512, bar);
+        bulk_load(st.wis, a.tab.wis + (size_t)h * 128, 512, bar);
+    }
     bulk_load(st.slot, a.tab.row_slot + (size_t)h * 128, 512, bar);
 }
 
@@ -313,9 +323,15 @@ __device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_
 // One decode step of one row-unit head page staged in shared memory
 // (App. C.3 steps 1-7; the Key-Row-Aware Dual-axis Fitting of Sec. 4.3 over
 // the non-pivot rows). `ok` and `refill` as for the pipeline's process().
-template <class Refill>
+//
+// MODE kReadout stops after the readout: it writes y and delta (delta_out) and
+// leaves the page untouched. MODE kWriteback takes delta from the stage (the
+// readout's, bit for bit), rebuilds Z exactly as the fused step does, and runs
+// steps 4-6; its y is not computed.
+template <int MODE, class Refill>
 __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Stage &st, float beta,
-                                            float *y_out, int fit_iters, bool ok, const Refill &refill) {
+                                            float *y_out, float *delta_out, int fit_iters, bool ok,
+                                            const Refill &refill) {
     uint16_t *page_r = (uint16_t *)st.page;
     uint16_t *page_c = (uint16_t *)(st.page + 256);
     // Row constants of the warp's band (warp-local).
@@ -337,7 +353,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         const float ki = st.k[i];
         S.rKap[sl] = ki * a;
         S.rBkp[sl] = __fdividef(beta * ki, a);
-        S.rQa[sl] = st.q[i] * a;
+        if (MODE != kWriteback) S.rQa[sl] = st.q[i] * a;
         S.rA[sl] = a;
         S.rMu[sl] = mu;
         S.rQm[sl] = qm;
@@ -345,7 +361,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         S.rMb[sl] = mb;
         S.rInfo[sl] = make_uint2(info, K);
     }
-    if (t.tid < 128) S.colM[t.tid] = 0u;
+    if (MODE != kReadout && t.tid < 128) S.colM[t.tid] = 0u;
     __syncwarp();
     // Step 1: Z = c_j q_ij (exact) or the FP16 value.
     uint64_t x2[8][4];
@@ -359,6 +375,32 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
 #pragma unroll
         for (int m = 0; m < 8; m++) load_pair(t, S, st.page, m, cd, x2[m]);
     }
+    float rs[16];
+    if constexpr (MODE == kWriteback) {
+        if (__syncthreads_or(!ok)) return false;
+        refill();
+        // Z += (beta k_i / a_i) delta_j with the readout's delta; row sums of |Z|.
+        uint64_t dl[4];
+        col_dup(st.v, t.l, dl);
+#pragma unroll
+        for (int p = 0; p < 4; p++) {
+            uint64_t blo, bhi;
+            row_pairs(S.rBkp, t, p, blo, bhi);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                x2[2 * p][c] = ffma2(blo, dl[c], x2[2 * p][c]);
+                x2[2 * p + 1][c] = ffma2(bhi, dl[c], x2[2 * p + 1][c]);
+            }
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                const uint64_t(&xm)[4] = x2[2 * p + h];
+                rs[4 * p + 2 * h] = (fabsf(f2lo(xm[0])) + fabsf(f2lo(xm[1]))) +
+                                    (fabsf(f2lo(xm[2])) + fabsf(f2lo(xm[3])));
+                rs[4 * p + 2 * h + 1] = (fabsf(f2hi(xm[0])) + fabsf(f2hi(xm[1]))) +
+                                        (fabsf(f2hi(xm[2])) + fabsf(f2hi(xm[3])));
+            }
+        }
+    } else {
     // Step 2a: retrieval u_j = sum_i k_i a_i Z_ij.
     {
         uint64_t ua[4] = {0, 0, 0, 0}, ub[4] = {0, 0, 0, 0};
@@ -382,11 +424,11 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
 #pragma unroll
         for (int wv = 0; wv < 8; wv++) s += S.red[wv * 128 + t.tid];
         S.colD[t.tid] = st.v[t.tid] - s;                   // delta_j = v_j - u_j
+        if (MODE == kReadout) delta_out[t.tid] = S.colD[t.tid];
     }
     refill();
     __syncthreads();
     // Step 2b-3: Z += (beta k_i / a_i) delta_j; readout partials q_i a_i Z_ij.
-    float rs[16];
     {
         uint64_t dl[4];
         col_dup(S.colD, t.l, dl);
@@ -403,18 +445,31 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
                 ya[c] = ffma2(qlo, x2[2 * p][c], ya[c]);
                 yb[c] = ffma2(qhi, x2[2 * p + 1][c], yb[c]);
             }
+            if (MODE == kFused) {
 #pragma unroll
-            for (int h = 0; h < 2; h++) {
-                const uint64_t(&xm)[4] = x2[2 * p + h];
-                rs[4 * p + 2 * h] = (fabsf(f2lo(xm[0])) + fabsf(f2lo(xm[1]))) +
-                                    (fabsf(f2lo(xm[2])) + fabsf(f2lo(xm[3])));
-                rs[4 * p + 2 * h + 1] = (fabsf(f2hi(xm[0])) + fabsf(f2hi(xm[1]))) +
-                                        (fabsf(f2hi(xm[2])) + fabsf(f2hi(xm[3])));
+                for (int h = 0; h < 2; h++) {
+                    const uint64_t(&xm)[4] = x2[2 * p + h];
+                    rs[4 * p + 2 * h] = (fabsf(f2lo(xm[0])) + fabsf(f2lo(xm[1]))) +
+                                        (fabsf(f2lo(xm[2])) + fabsf(f2lo(xm[3])));
+                    rs[4 * p + 2 * h + 1] = (fabsf(f2hi(xm[0])) + fabsf(f2hi(xm[1]))) +
+                                            (fabsf(f2hi(xm[2])) + fabsf(f2hi(xm[3])));
+                }
             }
         }
         const float v[4] = {pair_sum(fadd2(ya[0], yb[0])), pair_sum(fadd2(ya[1], yb[1])),
                             pair_sum(fadd2(ya[2], yb[2])), pair_sum(fadd2(ya[3], yb[3]))};
         cols_to_red(t, S.red, 2, v);
+    }
+    if (MODE == kReadout) {
+        __syncthreads();
+        if (t.tid < 128) {                              // the fused step's summation order
+            float s = S.red[(2 * 8) * 128 + t.tid];
+#pragma unroll
+            for (int wv = 1; wv < 8; wv++) s += S.red[(2 * 8 + wv) * 128 + t.tid];
+            y_out[t.tid] = s;
+        }
+        return true;
+    }
     }
     // Step 4: row factors r_i = m_i^(1/2) w_i^(-1/2) of the integer rows.
     {
@@ -474,7 +529,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         const float cc = fminf(fmaxf(c0, kF16Min), kF16Max);
         S.colC[t.tid] = cc;
         S.colG[t.tid] = __frcp_rn(cc);
-    } else {
+    } else if (MODE == kFused) {
         const int j = t.tid - 128;
         float s = S.red[(2 * 8) * 128 + j];
 #pragma unroll
@@ -537,6 +592,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     return true;
 }
 
+template <int MODE>
 __global__ void __launch_bounds__(kThreads, 2) decode_rows_kernel(DecodeArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     const T t;
@@ -555,16 +611,19 @@ __global__ void __launch_bounds__(kThreads, 2) decode_rows_kernel(DecodeArgs a) 
     __syncthreads();
     const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err};
     pipe::run(
-        p, S.bars, [&](int h, int b, int slot, int s) { issue(a, S, h, b, slot, s); },
+        p, S.bars, [&](int h, int b, int slot, int s) { issue<MODE>(a, S, h, b, slot, s); },
         [&](int h, int b, int, int s, bool ok, const auto &refill) {
-            const float beta = a.beta[(size_t)b * a.Hv + h];
+            const size_t u = (size_t)b * a.Hv + h;
+            const float beta = a.beta[u];
             const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
-            return decode_item(t, S, st, beta, a.y + ((size_t)b * a.Hv + h) * 128, a.fit_iters, ok,
-                               refill);
+            return decode_item<MODE>(t, S, st, beta, MODE == kWriteback ? nullptr : a.y + u * 128,
+                                     MODE == kReadout ? a.delta + u * 128 : nullptr, a.fit_iters, ok,
+                                     refill);
         },
         [&](int h, int slot, int s) {
-            bulk_store(a.pool + (uint64_t)slot * a.stride + S.hoff[h],
-                       S.stages + (size_t)s * a.stage_bytes, S.hbytes[h]);
+            if (MODE != kReadout)
+                bulk_store(a.pool + (uint64_t)slot * a.stride + S.hoff[h],
+                           S.stages + (size_t)s * a.stage_bytes, S.hbytes[h]);
         });
 }
 
@@ -574,6 +633,14 @@ stepq_status launch_decode_rows(const stepq_plan *p, int layer, uint8_t *pool, i
                                 const int32_t *slots, int B, const float *q, const float *k,
                                 const float *v, const float *beta, const float *gate, float *y,
                                 cudaStream_t s) {
+    return launch_decode_rows_mode(p, layer, pool, pool_slots, slots, B, q, k, v, beta, gate, y,
+                                   nullptr, rk::kFused, s);
+}
+
+stepq_status launch_decode_rows_mode(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
+                                     const int32_t *slots, int B, const float *q, const float *k,
+                                     const float *v, const float *beta, const float *gate, float *y,
+                                     float *delta, int mode, cudaStream_t s) {
     const int Hv = p->cfg.n_value_heads;
     if (Hv > rk::kMaxHv) return STEPQ_ERR_UNSUPPORTED;
     uint32_t maxb = 0;
@@ -590,6 +657,7 @@ stepq_status launch_decode_rows(const stepq_plan *p, int layer, uint8_t *pool, i
     a.items = B * Hv;
     a.tab = p->layer(layer);
     a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
+    a.delta = delta;
     a.err = device_error_word();
     a.page_region = (maxb + 127) / 128 * 128;
     a.stage_bytes = a.page_region + rk::kVecBytes;
@@ -599,15 +667,19 @@ stepq_status launch_decode_rows(const stepq_plan *p, int layer, uint8_t *pool, i
     a.n_stages = stages;
     a.fit_iters = p->cfg.fit_iters;
     const int smem = rk::kOffStages + stages * (int)a.stage_bytes;
-    if (cudaFuncSetAttribute((const void *)rk::decode_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem) != cudaSuccess)
+    const void *fn = mode == rk::kReadout     ? (const void *)rk::decode_rows_kernel<rk::kReadout>
+                     : mode == rk::kWriteback ? (const void *)rk::decode_rows_kernel<rk::kWriteback>
+                                              : (const void *)rk::decode_rows_kernel<rk::kFused>;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
         return STEPQ_ERR_CUDA;
     int dev = 0, sms = 1;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     int grid = 2 * (sms > 0 ? sms : 1);
     if (grid > a.items) grid = a.items;
-    rk::decode_rows_kernel<<<grid, kThreads, smem, s>>>(a);
+    if (mode == rk::kReadout) rk::decode_rows_kernel<rk::kReadout><<<grid, kThreads, smem, s>>>(a);
+    else if (mode == rk::kWriteback) rk::decode_rows_kernel<rk::kWriteback><<<grid, kThreads, smem, s>>>(a);
+    else rk::decode_rows_kernel<rk::kFused><<<grid, kThreads, smem, s>>>(a);
     return cudaGetLastError() == cudaSuccess ? STEPQ_OK : STEPQ_ERR_CUDA;
 }
 

@@ -32,7 +32,9 @@ def _setup(torch, name, kw, B, layer):
 
 
 @pytest.mark.parametrize("name,kw,layer", [("gqa", dict(n_pivots=3), 0),
-                                           ("pool", dict(layers=2, pool_slots=64, batch=16), 1)])
+                                           ("pool", dict(layers=2, pool_slots=64, batch=16), 1),
+                                           ("channel", {}, 0),
+                                           ("drift", dict(layers=2, pool_slots=32, batch=16), 1)])
 def test_readout_then_writeback_is_the_fused_step(torch, name, kw, layer):
     B = 16
     wl, plan, oplan, slots, pool_o = _setup(torch, name, kw, B, layer)
@@ -54,7 +56,9 @@ def test_readout_then_writeback_is_the_fused_step(torch, name, kw, layer):
     S_hat = O.pool_decode(oplan, pool_o, layer, slots).astype(np.float64)
     grp = wl.hv // wl.hk
     kk = np.repeat(inp.k.astype(np.float64), grp, axis=1)
-    u = np.einsum("bhi,bhij->bhj", kk * inp.gate.astype(np.float64)[..., None], S_hat)
+    g = inp.gate.astype(np.float64)
+    g = g if g.ndim == 3 else g[..., None]                 # per key channel or per head
+    u = np.einsum("bhi,bhij->bhj", kk * g, S_hat)
     d_o = inp.v - u
     err = np.abs(delta.cpu().numpy() - d_o).max(axis=-1)
     scale = np.abs(inp.v).max(axis=-1) + np.abs(u).max(axis=-1)
@@ -62,11 +66,12 @@ def test_readout_then_writeback_is_the_fused_step(torch, name, kw, layer):
     assert A.stepq_device_error() == 0
 
 
-def test_split_on_two_streams_over_steps(torch):
+@pytest.mark.parametrize("name,kw", [("gqa", dict(n_pivots=3)), ("channel", {})])
+def test_split_on_two_streams_over_steps(torch, name, kw):
     """Readout on the main stream, writeback on a side stream ordered by events,
     for 4 steps: the same pages and outputs as 4 fused steps."""
     B, layer, steps = 16, 0, 4
-    wl, plan, oplan, slots, pool_o = _setup(torch, "gqa", dict(n_pivots=3), B, layer)
+    wl, plan, oplan, slots, pool_o = _setup(torch, name, kw, B, layer)
     mp = W.model_params(wl)
     (pool0, slots_d) = to_dev(pool_o, slots)
     pool_f, pool_s = pool0.clone(), pool0.clone()
