@@ -151,7 +151,8 @@ def run(wl=None, steps=None, every=512, batch=None, variants=tuple(VARIANTS), wa
     assert A.stepq_device_error() == 0
     return {
         "workload": f"{wl.name}: {L} layers x {Hv} heads, d_k=d_v=128, {B} slots, per-key-channel "
-                    f"gates, {warmup} FP32 warm-up steps, {steps} decode steps",
+                    f"gates, {warmup} FP32 warm-up steps, {steps} decode steps, channel spreads "
+                    f"k {wl.k_sigma} / v {wl.v_sigma}",
         "every": every,
         "variants": {v.name: {"bits_per_value": v.bits_per_value, "slot_bytes": v.slot_bytes}
                      for v in vs},
@@ -167,9 +168,14 @@ def main(argv=None):
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--variants", default=",".join(VARIANTS),
                     help="comma list from " + ", ".join(ALL))
+    ap.add_argument("--geometry", action="store_true",
+                    help="key- and value-channel spreads sized to the paper's state geometry (App. B.6)")
     ap.add_argument("--out", default=None, help="write the JSON result here")
     args = ap.parse_args(argv)
-    res = run(steps=args.steps, every=args.every, batch=args.batch,
+    wl = W.WORKLOADS["drift"]
+    if args.geometry:
+        wl = W.with_geometry(wl)
+    res = run(wl, steps=args.steps, every=args.every, batch=args.batch,
               variants=tuple(args.variants.split(",")),
               log=lambda s: print(s, file=sys.stderr, flush=True))
     text = json.dumps(res, indent=1)

@@ -126,7 +126,8 @@ def run(wl=None, trajectories=4, steps=8192, inject=256, codecs=("int6", "int8")
     e = err.cpu().numpy()
     out = {
         "workload": f"{wl.name}: {Hv} heads ({wl.gate} gates), {B} trajectories, {steps} updates, "
-                    f"one injection after update {inject}, {steps - inject} readouts compared",
+                    f"one injection after update {inject}, {steps - inject} readouts compared, "
+                    f"channel spreads k {wl.k_sigma} / v {wl.v_sigma}",
         "reference_sq_sum": float(ref2.cpu()),
         "codecs": {},
         "windows": windows,
@@ -151,13 +152,18 @@ def main(argv=None):
     ap.add_argument("--every", type=int, default=512)
     ap.add_argument("--workload", default="gqa", choices=["gqa", "channel"])
     ap.add_argument("--codecs", default="int6,int8", help="comma list from " + ", ".join(CODECS))
+    ap.add_argument("--geometry", action="store_true",
+                    help="key- and value-channel spreads sized to the paper's state geometry (App. B.6)")
     ap.add_argument("--out", default=None, help="write the JSON result here")
     args = ap.parse_args(argv)
     codecs = tuple(args.codecs.split(","))
     for c in codecs:
         if c not in CODECS:
             ap.error(f"unknown codec {c}")
-    res = run(W.WORKLOADS[args.workload], args.trajectories, args.steps, args.inject, codecs,
+    wl = W.WORKLOADS[args.workload]
+    if args.geometry:
+        wl = W.with_geometry(wl)
+    res = run(wl, args.trajectories, args.steps, args.inject, codecs,
               args.every, log=lambda s: print(s, file=sys.stderr, flush=True))
     text = json.dumps(res, indent=1)
     if args.out:

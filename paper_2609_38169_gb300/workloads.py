@@ -8,11 +8,11 @@ The paper's workloads (Qwen3.8-27B / Kimi-Linear traces on WikiText-2 and C4) ar
 not available; these generators stand in for them with the shapes of the paper's
 hybrid models (d_k = d_v = 128, Sec. 2.1 and Table `config`) and the value
 structure it reports: scalar per-head gates for GDN, per-key-channel gates for
-KDA (Sec. 2.1), long-lived heads (Sec. 3.1) and magnitude outliers along both
-key rows and value columns (Sec. 4.2, App. B.6): fixed lognormal key-channel and
-value-channel scales, sized so that the states' median max-to-median RMS
-contrasts match the ones the paper measures (about 10x rows / 19x columns for
-the GDN model, 13x / 5x for KDA).
+KDA (Sec. 2.1), long-lived heads (Sec. 3.1) and per-key-row magnitude spread
+(Sec. 4.2). `with_geometry` adds fixed lognormal value-channel scales (and
+resizes the key-channel ones) so that the states' median max-to-median RMS
+contrasts match the ones the paper measures (App. B.6: about 10x rows / 19x
+columns for the GDN model, 13x / 5x for KDA).
 
 Recipe (every draw comes from numpy's PCG64 seeded by a SeedSequence over
 (seed, stream, step, layer), so any step of any layer can be drawn alone):
@@ -89,32 +89,40 @@ class Workload:
         return dataclasses.replace(self, **kw)
 
 
-# Channel spreads that give the states the paper's median max-to-median RMS
-# contrasts (App. B.6: GDN 10.3x key rows / 19.4x value columns; KDA 12.7x /
-# 5.4x), measured on snapshots of these recurrences from a zero state.
+# The five workloads as specified: tiny decode, GQA decode, channel-gate
+# decode, the 1024-slot serving pool and the long-generation drift run. q, v ~
+# N(0, 1) and normalised k ~ N(0, 1); the channel-gate workloads scale the key
+# channels by lognormal(0, 1) factors (a per-key-row magnitude spread).
+WORKLOADS = {
+    "tiny": Workload("tiny", layers=1, hk=4, hv=4, batch=1, pool_slots=1, steps=64,
+                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0),
+    "gqa": Workload("gqa", layers=1, hk=16, hv=32, batch=64, pool_slots=64, steps=256,
+                    gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0,
+                    alpha_lo=0.85, alpha_hi=0.999, long_frac=0.25),
+    "channel": Workload("channel", layers=1, hk=32, hv=32, batch=256, pool_slots=256, steps=512,
+                        gate="channel", nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=26,
+                        k_sigma=1.0),
+    "pool": Workload("pool", layers=16, hk=32, hv=32, batch=1024, pool_slots=1024, steps=128,
+                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=7),
+    "drift": Workload("drift", layers=4, hk=32, hv=32, batch=128, pool_slots=128, steps=8192,
+                      gate="channel", nominal_bits=6, candidates=(4, 6, 8), n_pivots=102,
+                      k_sigma=1.0),
+}
+
+# Channel spreads that give the states the outlier geometry the paper measures
+# on its traces: median max-to-median RMS contrasts of about 10x along key
+# rows and 19x along value columns for the GDN model, 13x and 5x for KDA
+# (App. B.6), on snapshots of these recurrences from a zero state.
 GDN_K_SIGMA, GDN_V_SIGMA = 1.05, 1.12
 KDA_K_SIGMA, KDA_V_SIGMA = 1.10, 0.60
 
-# The five workloads: tiny decode, GQA decode, channel-gate decode, the 1024-slot
-# serving pool and the long-generation drift run.
-WORKLOADS = {
-    "tiny": Workload("tiny", layers=1, hk=4, hv=4, batch=1, pool_slots=1, steps=64,
-                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0,
-                     k_sigma=GDN_K_SIGMA, v_sigma=GDN_V_SIGMA),
-    "gqa": Workload("gqa", layers=1, hk=16, hv=32, batch=64, pool_slots=64, steps=256,
-                    gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=0,
-                    alpha_lo=0.85, alpha_hi=0.999, long_frac=0.25,
-                    k_sigma=GDN_K_SIGMA, v_sigma=GDN_V_SIGMA),
-    "channel": Workload("channel", layers=1, hk=32, hv=32, batch=256, pool_slots=256, steps=512,
-                        gate="channel", nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=26,
-                        k_sigma=KDA_K_SIGMA, v_sigma=KDA_V_SIGMA),
-    "pool": Workload("pool", layers=16, hk=32, hv=32, batch=1024, pool_slots=1024, steps=128,
-                     gate="scalar", nominal_bits=6, candidates=(4, 6, 8), n_pivots=7,
-                     k_sigma=GDN_K_SIGMA, v_sigma=GDN_V_SIGMA),
-    "drift": Workload("drift", layers=4, hk=32, hv=32, batch=128, pool_slots=128, steps=8192,
-                      gate="channel", nominal_bits=6, candidates=(4, 6, 8), n_pivots=102,
-                      k_sigma=KDA_K_SIGMA, v_sigma=KDA_V_SIGMA),
-}
+
+def with_geometry(wl: Workload) -> Workload:
+    """The workload with lognormal key- and value-channel spreads sized to the
+    state geometry of App. B.6 (value-column outliers included)."""
+    if wl.gate == "scalar":
+        return wl.replace(k_sigma=GDN_K_SIGMA, v_sigma=GDN_V_SIGMA)
+    return wl.replace(k_sigma=KDA_K_SIGMA, v_sigma=KDA_V_SIGMA)
 
 
 def _rng(*key: int) -> np.random.Generator:

@@ -5,7 +5,12 @@ States: an all-zero state (every scale at its FP16 floor, codes 0), states
 scaled by 1e9 (the clip-free column start exceeds the FP16 range, so the
 codes take the clamped path), states scaled by 1e-12 (row factors at the
 FP16 floor) and a state of tiny values with a few large outliers. Each runs
-two teacher-forced decode steps under the parity rules of gpu_helpers.
+two teacher-forced decode steps under the parity rules of gpu_helpers, with
+one addition for FP16 pivot values: the tile is fp32 (the oracle rounds an
+fp64 result once), so a pivot value that is the small difference of large
+terms (the retrieval's sum, the update's two parts) may differ by the fp32
+rounding of those terms, 2^-21 of their magnitude, even when that exceeds one
+FP16 ulp of the result.
 """
 import numpy as np
 import pytest
@@ -39,6 +44,22 @@ def _degenerate_states(wl, B=4):
     return S.astype(np.float32)
 
 
+def _update_term_bound(wl, S_hat, inp):
+    """Absolute fp32 rounding allowance of the updated state X = D S + beta k
+    (v - k^T D S)^T: 2^-21 of the magnitudes that enter it, |D S_ij| +
+    |beta k_i| (|v_j| + sum_i' |k_i' (D S)_i'j|); the retrieval's fp32 sum
+    carries the rounding of its largest terms into delta_j, and the update's
+    terms may nearly cancel. S_hat: [B][Hv][128][128] decoded state."""
+    grp = wl.hv // wl.hk
+    k = np.repeat(inp.k.astype(np.float64), grp, axis=1)
+    g = inp.gate.astype(np.float64)
+    g = g if g.ndim == 3 else np.broadcast_to(g[..., None], k.shape)
+    DS = g[..., None] * S_hat
+    dmag = np.abs(inp.v.astype(np.float64)) + np.einsum("bhi,bhij->bhj", np.abs(k), np.abs(DS))
+    T = np.abs(DS) + np.abs(inp.beta.astype(np.float64)[..., None, None] * k[..., None]) * dmag[:, :, None, :]
+    return 2.0 ** -21 * T
+
+
 def _teacher_forced(torch, wl, S, steps=2):
     cfg, plan, oplan, _ = plans(wl)
     mp = W.model_params(wl)
@@ -54,13 +75,14 @@ def _teacher_forced(torch, wl, S, steps=2):
     for step in range(steps):
         inp = W.step_inputs(wl, mp, W.STREAM_DECODE, step, 0, batch=B)
         pool_d.copy_(torch.from_numpy(pool_o))
+        tol = _update_term_bound(wl, O.pool_decode(oplan, pool_o, 0, slots).astype(np.float64), inp)
         q, k, v, beta, gate = to_dev(inp.q, inp.k, inp.v, inp.beta, inp.gate)
         y_d = torch.empty((B, wl.hv, 128), dtype=torch.float32, device="cuda")
         A.stepq_decode_step(plan, 0, pool_d, slots_d, q, k, v, beta, gate, y_d)
         y_o = O.pool_step(oplan, pool_o, 0, slots, inp)
         assert np.isfinite(y_d.cpu().numpy()).all()
         compare_y(t, y_d.cpu().numpy(), y_o)
-        compare_pools(t, pool_d.cpu().numpy(), pool_o, oplan, 0, slots)
+        compare_pools(t, pool_d.cpu().numpy(), pool_o, oplan, 0, slots, piv_tol=tol)
     return t
 
 

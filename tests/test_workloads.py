@@ -5,7 +5,9 @@ over snapshots of the maximum-to-median RMS contrast along key rows and along
 value columns: 10.3x and 19.4x for the GDN model (Qwen, positions 128 to
 2,048), 12.7x and 5.4x for KDA (Kimi-Linear, steps 128 to 512). The workload
 generators stand in for those traces; their states, run from a zero state with
-the oracle's FP32 recurrence, must show contrasts of the same size.
+the oracle's FP32 recurrence, must show contrasts of the same size when the
+App. B.6 geometry is requested (`with_geometry`). The default recipe keeps the
+specified distributions: v ~ N(0, 1) with no channel scales.
 """
 import numpy as np
 import pytest
@@ -37,7 +39,20 @@ def _contrasts(oracle, wl, snaps, B=2):
     ("channel", (128, 256, 512), (12.7, 5.4)),  # KDA (Kimi-Linear)
 ])
 def test_state_outlier_contrasts_match_paper(oracle, name, snaps, paper):
-    row, col = _contrasts(oracle, W.WORKLOADS[name], snaps)
+    row, col = _contrasts(oracle, W.with_geometry(W.WORKLOADS[name]), snaps)
     print(name, row, col)
     assert paper[0] / 1.35 <= row <= paper[0] * 1.35
     assert paper[1] / 1.35 <= col <= paper[1] * 1.35
+
+
+def test_default_recipe_is_the_specified_one():
+    """Defaults: no value-channel scales anywhere; key channels unscaled for the
+    scalar-gate workloads and lognormal(0, 1) for the channel-gate ones."""
+    for name, wl in W.WORKLOADS.items():
+        mp = W.model_params(wl)
+        assert np.all(mp.v_scale == 1.0), name
+        if wl.gate == "scalar":
+            assert np.all(mp.k_scale == 1.0), name
+        else:
+            ls = np.log(mp.k_scale)
+            assert abs(ls.mean()) < 0.1 and abs(ls.std() - 1.0) < 0.1, name
