@@ -7,6 +7,7 @@ generators), resident on the device, and timed with CUDA events after warm-up.
     python -m paper_2609_38169_gb300.measure rows [--slots 1024] [--bits 6]
     python -m paper_2609_38169_gb300.measure prefill [--slots 128] [--tokens 512]
     python -m paper_2609_38169_gb300.measure split [--slots 1024] [--layers 16]
+    python -m paper_2609_38169_gb300.measure calib [--workload pool]
 """
 from __future__ import annotations
 
@@ -215,6 +216,31 @@ def split(slots=1024, layers=16):
     return out
 
 
+def calib(name="pool", layers=None):
+    """The calibration statistics of App. A.3 on the device: omega and ell over
+    the calibration stream, then the candidate distortions of states sampled
+    from the FP32 recurrence (twice for row units, with pivots held out)."""
+    import time
+    import torch
+    dev = torch.device("cuda")
+    wl = W.WORKLOADS[name]
+    if layers is not None:
+        wl = wl.replace(layers=layers)
+    cfg = A.Config.from_workload(wl)
+    wl1 = wl.replace(layers=1)
+    A.calibrate(A.Config.from_workload(wl1), wl1, dev, seqs=2, steps=8, device_inputs=True)   # warm-up
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    st = A.calibrate(cfg, wl, dev, device_inputs=True)
+    torch.cuda.synchronize()
+    t = time.perf_counter() - t0
+    assert A.stepq_device_error() == 0
+    return {"metric": "calibration statistics on the device", "unit": "s", "value": t,
+            "workload": f"{name}: {wl.layers} layers x {wl.hv} heads, {wl.calib_seqs} sequences x "
+                        f"{wl.calib_steps} tokens, states sampled every {wl.calib_every} updates",
+            "calibration_tokens": int(st.n_tokens), "sampled_states_per_layer": int(st.n_samples)}
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     sub = ap.add_subparsers(dest="what", required=True)
@@ -225,6 +251,8 @@ def main(argv=None):
     p.add_argument("--slots", type=int, default=128)
     p.add_argument("--tokens", type=int, default=512)
     p.add_argument("--workload", default="gqa", choices=["gqa", "channel", "pool"])
+    cb = sub.add_parser("calib")
+    cb.add_argument("--workload", default="pool", choices=["gqa", "channel", "pool", "drift"])
     sp = sub.add_parser("split")
     sp.add_argument("--slots", type=int, default=1024)
     sp.add_argument("--layers", type=int, default=16)
@@ -233,6 +261,8 @@ def main(argv=None):
         res = rows(args.slots, args.bits)
     elif args.what == "split":
         res = split(args.slots, args.layers)
+    elif args.what == "calib":
+        res = calib(args.workload)
     else:
         res = prefill(args.slots, args.tokens, args.workload)
     print(json.dumps(res))

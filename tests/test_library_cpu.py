@@ -160,7 +160,7 @@ def test_feedback_cli():
 def test_measure_cli():
     """The secondary-measurement module parses its subcommands (no device work)."""
     from paper_2609_38169_gb300 import measure
-    for argv in (["--help"], ["rows", "--help"], ["prefill", "--help"], ["split", "--help"]):
+    for argv in (["--help"], ["rows", "--help"], ["prefill", "--help"], ["split", "--help"], ["calib", "--help"]):
         with pytest.raises(SystemExit) as e:
             measure.main(argv)
         assert e.value.code == 0
