@@ -152,13 +152,14 @@ __device__ __forceinline__ void store_row(uint8_t *row, int l, uint32_t f0, uint
         const uint32_t lo = __byte_perm(f0, f1, 0x0040), hi = __byte_perm(f2, f3, 0x0040);
         ((uint32_t *)row)[l] = __byte_perm(lo, hi, 0x5410);
     } else if (B == 6) {
-        // Lane l holds bits 24l..24l+23 of the row; lane t < 24 assembles word t
-        // from lanes floor(4t/3) and the next (offset 0, 8 or 16 bits).
+        // Lane l writes its 24 bits as bytes 3l .. 3l + 2 of the row: one aligned
+        // 16-bit store and one byte store (which is which depends on l's parity).
         constexpr uint32_t K = kMagicBits + (kMagicBits << 6) + (kMagicBits << 12) + (kMagicBits << 18);
         const uint32_t v = (f0 + (f1 << 6) + (f2 << 12) + (f3 << 18) - K) & 0xFFFFFFu;
-        const int lt = min(l, 23), l0 = (4 * lt) / 3, off = 32 * lt - 24 * l0;
-        const uint32_t a = __shfl_sync(0xffffffffu, v, l0), b = __shfl_sync(0xffffffffu, v, l0 + 1);
-        if (l < 24) ((uint32_t *)row)[l] = (a >> off) | (b << (24 - off));
+        const int odd = l & 1;
+        uint8_t *p = row + 3 * l;
+        *(uint16_t *)(p + odd) = (uint16_t)(odd ? v >> 8 : v);
+        p[odd ? 0 : 2] = (uint8_t)(odd ? v : v >> 16);
     } else {
         constexpr uint32_t K = kMagicBits + (kMagicBits << 4) + (kMagicBits << 8) + (kMagicBits << 12);
         ((uint16_t *)row)[l] = (uint16_t)(f0 + (f1 << 4) + (f2 << 8) + (f3 << 12) - K);
