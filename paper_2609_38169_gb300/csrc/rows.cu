@@ -144,10 +144,12 @@ __device__ __forceinline__ void store_segment(uint8_t *row, int b, int l, uint32
     } else if (b == 2) {
         row[l] = (uint8_t)v;
     } else {
-        // 24 bits per lane: lanes 4g..4g+2 each store one of the words 3g..3g+2
-        const uint32_t nb = __shfl_down_sync(0xffffffffu, v, 1);
-        const int j = l & 3;
-        if (j < 3) ((uint32_t *)row)[3 * (l >> 2) + j] = (v >> (8 * j)) | (nb << (24 - 8 * j));
+        // 24 bits per lane, bytes 3l .. 3l + 2: one aligned 16-bit store and one
+        // byte store (which is which depends on l's parity)
+        const int odd = l & 1;
+        uint8_t *p = row + 3 * l;
+        *(uint16_t *)(p + odd) = (uint16_t)(odd ? v >> 8 : v);
+        p[odd ? 0 : 2] = (uint8_t)(odd ? v : v >> 16);
     }
 }
 
