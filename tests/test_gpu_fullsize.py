@@ -1,10 +1,16 @@
-"""Full-size parity on the 1024-slot serving pool, in the launch configuration the
-timing script uses (16 layers x 32 heads, all 1024 slots in a random
-permutation, one launch per layer-step).
+"""Full-size parity in the launch configuration of each workload's timing: every
+active slot of the pool in a random permutation, one launch per layer-step.
 
-The whole 6.8 GB pool is packed on the GPU; a sample of (slot, layer, head)
-units gets pages packed by the oracle from its own states instead, so the
-oracle can step exactly those units one by one and compare outputs and pages.
+- the 1024-slot serving pool (16 layers x 32 heads, head units, the bench's
+  workload);
+- the channel-gate decode workload (1 layer x 32 heads, 256 slots, row units
+  at 4 bits);
+- the drift workload's pool (4 layers x 32 heads, 128 slots, row units at 6
+  bits).
+
+The whole pool is packed on the GPU; a sample of (slot, layer, head) units gets
+pages packed by the oracle from its own states instead, so the oracle can step
+exactly those units one by one and compare outputs and pages.
 """
 import numpy as np
 import pytest
@@ -17,11 +23,25 @@ from gpu_helpers import Tally, compare_head, compare_y
 pytestmark = pytest.mark.gpu
 
 
-def test_pool_full_size_sampled(tmp_path):
+def _sample_heads(oplan, layer, Hv, rng):
+    """Every FP16 pivot head and one head per width (head units), or the heads
+    holding pivot rows (row units, at most four), plus six random heads."""
+    if oplan.unit_kind == O.UNIT_HEAD:
+        bits = oplan.unit_bits[layer * Hv:(layer + 1) * Hv]
+        heads = list(np.flatnonzero(bits == 16)) + [int(np.flatnonzero(bits == b)[0])
+                                                    for b in (2, 4, 6, 8) if np.any(bits == b)]
+    else:
+        rows = oplan.unit_bits.reshape(oplan.n_layers, Hv, 128)[layer]
+        heads = list(np.flatnonzero((rows == 16).any(axis=1))[:4])
+    return [int(h) for h in heads] + [int(h) for h in rng.choice(Hv, 6, replace=False)]
+
+
+@pytest.mark.parametrize("name,layers", [("pool", [0, 7, 15]), ("channel", [0]), ("drift", [0, 3])])
+def test_full_size_sampled(name, layers):
     torch = pytest.importorskip("torch")
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
-    wl = W.WORKLOADS["pool"]
+    wl = W.WORKLOADS[name]
     st = O.calibrate(wl, seqs=2, steps=8)
     oplan = O.plan_from_stats(wl, st)
     cfg = A.Config.from_workload(wl)
@@ -43,19 +63,14 @@ def test_pool_full_size_sampled(tmp_path):
     slots = W.slot_permutation(wl)
     slots_d = torch.from_numpy(slots).to(dev)
 
-    # sampled units: every pivot head, every bit width, spread over layers/slots
     rng = np.random.default_rng(7)
-    layers = [0, 7, 15]
     units = {}
     for layer in layers:
-        bits = oplan.unit_bits[layer * Hv:(layer + 1) * Hv]
-        heads = list(np.flatnonzero(bits == 16)) + [int(np.flatnonzero(bits == b)[0])
-                                                    for b in (4, 6, 8) if np.any(bits == b)]
-        heads += list(rng.choice(Hv, 6, replace=False))
-        units[layer] = [(int(rng.integers(B)), int(h)) for h in heads] + [(0, 0), (B - 1, Hv - 1)]
+        heads = _sample_heads(oplan, layer, Hv, rng)
+        units[layer] = [(int(rng.integers(B)), h) for h in heads] + [(0, 0), (B - 1, Hv - 1)]
     mp = W.model_params(wl)
+    grp = Hv // Hk
     t = Tally()
-    pool_host = None
     for layer in layers:
         rb_layer = oplan.layer_row_bits(layer)
         offs = oplan.layer_head_off(layer)
@@ -78,7 +93,6 @@ def test_pool_full_size_sampled(tmp_path):
         y_h = y.cpu().numpy()
         assert np.isfinite(y_h).all()
         for (b, h), page in pages.items():
-            grp = Hv // Hk
             page_o, y_o = O.step_head(page, oplan.unit_kind, rb_layer[h], w_layer[h],
                                       inp.q[b, h // grp], inp.k[b, h // grp], inp.v[b, h],
                                       inp.beta[b, h], inp.gate[b, h], wl.fit_iters)
@@ -86,5 +100,5 @@ def test_pool_full_size_sampled(tmp_path):
             page_g = pool[base:base + int(nb[h])].cpu().numpy()
             compare_y(t, y_h[b, h], y_o)
             compare_head(t, page_g, page_o, oplan.unit_kind, rb_layer[h], w_layer[h])
-    print(t.summary())
+    print(name, t.summary())
     t.check()
