@@ -34,6 +34,7 @@ def _slots(wl, batch, seed=11):
     ("channel", {}, 24),
     ("gqa", dict(n_pivots=3), 8),
     ("channel", dict(nominal_bits=6, candidates=(4, 6, 8), n_pivots=40), 8),
+    ("gqa", dict(nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=2), 16),    # 2-bit heads
 ])
 def test_quantize_dequantize_pool(torch, name, kw, batch):
     """Pack fp32 states (App. C.3 steps 4-6) and unpack them again."""
@@ -66,6 +67,8 @@ def test_quantize_dequantize_pool(torch, name, kw, batch):
     ("gqa", dict(n_pivots=3), 16, 4),
     ("channel", dict(nominal_bits=6, candidates=(4, 6, 8), n_pivots=40), 16, 4),
     ("tiny", dict(fit_iters=3), 1, 8),
+    ("gqa", dict(nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=2), 16, 4),  # 2-bit heads
+    ("channel", dict(fit_iters=2), 16, 3),                                     # row units, two LS passes
 ])
 def test_decode_step_teacher_forced(torch, name, kw, batch, steps):
     """App. C.3 steps 1-7 against the oracle, step by step."""

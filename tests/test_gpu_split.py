@@ -34,7 +34,8 @@ def _setup(torch, name, kw, B, layer):
 @pytest.mark.parametrize("name,kw,layer", [("gqa", dict(n_pivots=3), 0),
                                            ("pool", dict(layers=2, pool_slots=64, batch=16), 1),
                                            ("channel", {}, 0),
-                                           ("drift", dict(layers=2, pool_slots=32, batch=16), 1)])
+                                           ("drift", dict(layers=2, pool_slots=32, batch=16), 1),
+                                          ("gqa", dict(nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=2), 0)])
 def test_readout_then_writeback_is_the_fused_step(torch, name, kw, layer):
     B = 16
     wl, plan, oplan, slots, pool_o = _setup(torch, name, kw, B, layer)
