@@ -317,28 +317,37 @@ def main():
 
     # ---- end to end through the public API with host buffers ----
     # Every step copies each layer's inputs from pinned host memory and reads
-    # every layer's y back. The copies run on their own streams, one layer
-    # ahead of / behind the kernel that uses them (two device input buffers,
-    # ordered by events), so they overlap the decode kernels; the step ends
-    # when the last y has reached the host.
+    # every layer's y back. The copies run on their own streams, up to two
+    # layers ahead of / one behind the kernel that uses them (three device
+    # input buffers, ordered by events), so they overlap the decode kernels;
+    # the step ends when the last y has reached the host.
     h_in = []
     for layer in range(L):
         h_in.append([x.cpu().pin_memory() for x in inputs[0][layer]])
-    d_in = [[torch.empty_like(x) for x in inputs[0][0]] for _ in range(2)]
+    n_buf = 3
+    d_in = [[torch.empty_like(x) for x in inputs[0][0]] for _ in range(n_buf)]
     h_y = torch.empty((L, B, Hv, 128), dtype=torch.float32).pin_memory()
     h2d = sum(x.numel() * x.element_size() for row in h_in for x in row)
     d2h = h_y.numel() * 4
     h2d_stream, d2h_stream = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
-    buf_free = [torch.cuda.Event() for _ in range(2)]
-    copied = [torch.cuda.Event() for _ in range(2)]
+    buf_free = [torch.cuda.Event() for _ in range(n_buf)]
+    copied = [torch.cuda.Event() for _ in range(n_buf)]
     y_done = [torch.cuda.Event() for _ in range(L)]
     y_read = [torch.cuda.Event() for _ in range(L)]
+    lookahead = 2
+    step_done = [torch.cuda.Event() for _ in range(lookahead + 1)]
     for e in buf_free + y_read:
         e.record(stream)
 
     def step_e2e(s):
+        # At most `lookahead` steps in flight, as a serving loop keeps them. An
+        # unbounded loop fills the launch queue, and the host then blocks on the
+        # decode stream while the next layers' input copies, on their own
+        # stream, are not yet issued.
+        if s >= lookahead:
+            step_done[(s - lookahead) % (lookahead + 1)].synchronize()
         for layer in range(L):
-            nb = (s * L + layer) % 2
+            nb = (s * L + layer) % n_buf
             h2d_stream.wait_event(buf_free[nb])         # the kernel that last read this buffer
             with torch.cuda.stream(h2d_stream):
                 for dst, src in zip(d_in[nb], h_in[layer]):
@@ -356,6 +365,7 @@ def main():
                 h_y[layer].copy_(y[layer], non_blocking=True)
                 y_read[layer].record(d2h_stream)
         stream.wait_event(y_read[L - 1])                # the step ends with y on the host
+        step_done[s % (lookahead + 1)].record(stream)
 
     e2e_steps = max(3, args.steps // 2)
     e2e_ms, _ = timed(step_e2e, e2e_steps, 2, name="stepq_e2e")
