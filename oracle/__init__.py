@@ -49,7 +49,11 @@ _lib = None
 def lib():
     global _lib
     if _lib is None:
-        _lib = C.CDLL(build())
+        # STEPQ_ORACLE_LIB names a separately built copy of this library; the
+        # planted-mistake tests (tests/test_oracle_mutations.py) run the pins
+        # against mutated copies this way.
+        path = os.environ.get("STEPQ_ORACLE_LIB")
+        _lib = C.CDLL(path if path else build())
         _declare(_lib)
     return _lib
 
@@ -91,6 +95,7 @@ def _declare(L):
         "or_lifetime_weight": (D_, [D_, I]),
         "or_allocate_dp": (I, [I, I, P, LL, P, P]),
         "or_allocate_lagrangian": (I, [I, I, P, LL, P, P]),
+        "or_lagrangian_multiplier": (D_, [I, I, P, LL, P]),
         "or_select_pivots": (I, [I, I, I, P, I, P, P, I, P]),
         "or_allocate": (I, [I, I, I, P, I, P, P, P, P]),
         "or_layout": (I, [I, I, I, P, P, P, P]),
@@ -339,6 +344,15 @@ def allocate_lagrangian(cost, cands, budget_bits):
     c = np.ascontiguousarray(cands, np.int32)
     rc = lib().or_allocate_lagrangian(U, K, _p(c), int(budget_bits), _p(cost), _p(ch))
     return None if rc else ch
+
+
+def lagrangian_multiplier(cost, cands, budget_bits):
+    """The Lagrangian relaxation's multiplier (None if nothing fits)."""
+    cost = np.ascontiguousarray(cost, np.float64)
+    U, K = cost.shape
+    c = np.ascontiguousarray(cands, np.int32)
+    lam = lib().or_lagrangian_multiplier(U, K, _p(c), int(budget_bits), _p(cost))
+    return None if lam < 0 else lam
 
 
 def select_pivots(unit_kind, cands, nominal, L, dist, n_pivots):

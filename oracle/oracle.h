@@ -93,6 +93,8 @@ int or_allocate_dp(int n_units, int n_cand, const int *cands, long long capacity
                    const double *cost, int8_t *choice);
 int or_allocate_lagrangian(int n_units, int n_cand, const int *cands, long long budget_bits,
                            const double *cost, int8_t *choice);
+double or_lagrangian_multiplier(int n_units, int n_cand, const int *cands, long long budget_bits,
+                                const double *cost);
 int or_select_pivots(int unit_kind, int n_units, int n_cand, const int *cands, int nominal,
                      const double *L, const double *dist, int n_pivots, uint8_t *pivot);
 int or_allocate(int unit_kind, int n_units, int n_cand, const int *cands, int nominal,

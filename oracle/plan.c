@@ -125,12 +125,8 @@ static long long lagr_pick(int n_units, int n_cand, const int *asc, const int *c
     return bits;
 }
 
-/* Lagrangian allocation with a shared multiplier and a discrete repair
- * (App. C.2): minimise sum_u cost[u][k_u] s.t. sum_u cands[k_u] <= budget. */
-int or_allocate_lagrangian(int n_units, int n_cand, const int *cands, long long budget,
-                           const double *cost, int8_t *choice)
+static void ascending(int n_cand, const int *cands, int *asc)
 {
-    int asc[8];
     for (int k = 0; k < n_cand; k++)
         asc[k] = k;
     for (int a = 0; a < n_cand; a++)
@@ -138,16 +134,30 @@ int or_allocate_lagrangian(int n_units, int n_cand, const int *cands, long long 
             if (cands[asc[b]] < cands[asc[a]]) {
                 int t = asc[a]; asc[a] = asc[b]; asc[b] = t;
             }
+}
+
+/* The shared multiplier of the Lagrangian relaxation (App. C.2): 0 if the
+ * unconstrained choice fits the budget, else the smallest lambda (bisection,
+ * 60 steps in fp64) whose per-unit choices argmin_k cost[u][k] + lambda cands[k]
+ * (ties to the narrower code) fit. Returns -1 if no choice fits. */
+double or_lagrangian_multiplier(int n_units, int n_cand, const int *cands, long long budget,
+                                const double *cost)
+{
+    int asc[8];
+    ascending(n_cand, cands, asc);
     if ((long long)cands[asc[0]] * n_units > budget)
-        return -1;
+        return -1.0;
+    int8_t *choice = malloc((size_t)(n_units > 0 ? n_units : 1));
     double lam = 0.0;
     if (lagr_pick(n_units, n_cand, asc, cands, cost, 0.0, choice) > budget) {
         double lo = 0.0, hi = 1.0;
         int guard = 0;
         while (lagr_pick(n_units, n_cand, asc, cands, cost, hi, choice) > budget) {
             hi *= 2.0;
-            if (++guard > 2000 || !isfinite(hi))
-                return -1;
+            if (++guard > 2000 || !isfinite(hi)) {
+                free(choice);
+                return -1.0;
+            }
         }
         for (int it = 0; it < 60; it++) {
             double mid = 0.5 * (lo + hi);
@@ -158,6 +168,20 @@ int or_allocate_lagrangian(int n_units, int n_cand, const int *cands, long long 
         }
         lam = hi;
     }
+    free(choice);
+    return lam;
+}
+
+/* Lagrangian allocation with a shared multiplier and a discrete repair
+ * (App. C.2): minimise sum_u cost[u][k_u] s.t. sum_u cands[k_u] <= budget. */
+int or_allocate_lagrangian(int n_units, int n_cand, const int *cands, long long budget,
+                           const double *cost, int8_t *choice)
+{
+    int asc[8];
+    ascending(n_cand, cands, asc);
+    double lam = or_lagrangian_multiplier(n_units, n_cand, cands, budget, cost);
+    if (lam < 0.0)
+        return -1;
     long long bits = lagr_pick(n_units, n_cand, asc, cands, cost, lam, choice);
     long long slack = budget - bits;
     for (;;) {

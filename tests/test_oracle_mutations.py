@@ -1,0 +1,134 @@
+"""Planted mistakes in the oracle (CPU only).
+
+Each mutant is a copy of the oracle's C sources with one plausible error in
+one function: a flipped sign, a dropped term or factor, a wrong exponent,
+rounding mode, bias or index, an off-by-one budget or order. It is compiled on
+its own, and the oracle's pin tests (which check it against the paper's
+printed values, closed forms, brute force and invariants, never against the
+CUDA library) run against it in a subprocess. Every mutant must fail at least
+one pin. A control run of an unmodified copy must pass them all.
+"""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+ORACLE = os.path.join(ROOT, "oracle")
+SOURCES = ["numerics.c", "recurrence.c", "codec.c", "plan.c", "batch.c", "calib.c"]
+PINS = ["tests/test_oracle_numerics.py", "tests/test_oracle_recurrence.py", "tests/test_oracle_codec.py",
+        "tests/test_oracle_plan.py", "tests/test_oracle_step.py"]
+
+DELTA_W = ("            S[i * OR_D + j] = (float)(P[i * OR_D + j] +\n"
+           "                                      (double)beta * (double)k[i] * ((double)v[j] - u[j]));")
+STEP_W = ("            X[i * OR_D + j] = (float)(S[i * OR_D + j] +\n"
+          "                                      (double)beta * (double)k[i] * ((double)v[j] - u[j]));\n"
+          "    for (int j = 0; j < OR_D; j++) {                           /* readout before requantization */")
+STEP_Y = ("    for (int j = 0; j < OR_D; j++) {                           /* readout before requantization */\n"
+          "        double acc = 0.0;\n"
+          "        for (int i = 0; i < OR_D; i++)\n"
+          "            acc += (double)q[i] * (double)X[i * OR_D + j];")
+INTB_W = ("            X[i * OR_D + j] = (float)(S[i * OR_D + j] +\n"
+          "                                      (double)beta * (double)k[i] * ((double)v[j] - u[j]));\n"
+          "    for (int j = 0; j < OR_D; j++) {\n"
+          "        double acc = 0.0;")
+READOUT = ("    for (int j = 0; j < OR_D; j++) {                              /* readout S^T q */\n"
+           "        double acc = 0.0;\n"
+           "        for (int i = 0; i < OR_D; i++)\n"
+           "            acc += (double)q[i] * (double)S[i * OR_D + j];")
+
+# (id, file, original text, mutated text)
+MUTANTS = [
+    ("delta_sign", "recurrence.c", DELTA_W, DELTA_W.replace("((double)v[j] - u[j])", "(u[j] - (double)v[j])")),
+    ("retrieval_ungated", "recurrence.c", "            acc += (double)k[i] * P[i * OR_D + j];",
+     "            acc += (double)k[i] * (double)S[i * OR_D + j];"),
+    ("readout_before_update", "recurrence.c", READOUT,
+     READOUT.replace("(double)q[i] * (double)S[i * OR_D + j]", "(double)q[i] * P[i * OR_D + j]")),
+    ("row_impact_gate_dropped", "recurrence.c",
+     "        g[i] = d * ((double)q[i] - (double)beta * (double)k[i] * kq);",
+     "        g[i] = ((double)q[i] - (double)beta * (double)k[i] * kq);"),
+    ("exact_read_own_state", "recurrence.c",
+     "            acc += (double)k[i] * (d * (double)Sref[i * OR_D + j]);",
+     "            acc += (double)k[i] * (d * (double)S[i * OR_D + j]);"),
+    ("step_delta_sign", "codec.c", STEP_W, STEP_W.replace("((double)v[j] - u[j])", "(u[j] - (double)v[j])")),
+    ("step_readout_source", "codec.c", STEP_Y,
+     STEP_Y.replace("(double)q[i] * (double)X[i * OR_D + j]", "(double)k[i] * (double)X[i * OR_D + j]")),
+    ("intb_step_delta_sign", "codec.c", INTB_W, INTB_W.replace("((double)v[j] - u[j])", "(u[j] - (double)v[j])")),
+    ("ls_weight_w_not_w2", "codec.c", "                double w2 = (double)w[i] * (double)w[i];",
+     "                double w2 = (double)w[i];"),
+    ("row_factor_exponent", "codec.c", "        float wis = (float)(1.0 / sqrt((double)w[i]));",
+     "        float wis = (float)sqrt((double)w[i]);"),
+    ("column_start_without_mu", "codec.c",
+     "                float a = mul32(mul32(fabsf(X[i * OR_D + j]), rho[i]), mu[i]);",
+     "                float a = mul32(fabsf(X[i * OR_D + j]), rho[i]);"),
+    ("codes_truncated", "codec.c",
+     "static double rne_prod(float a, float b) { return rint((double)a * (double)b); }",
+     "static double rne_prod(float a, float b) { return trunc((double)a * (double)b); }"),
+    ("offset_binary_bias", "codec.c",
+     "            put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1))));",
+     "            put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1)) - 1));"),
+    ("final_codes_unrounded_c", "codec.c", "        gamma[j] = (float)(1.0 / c16[j]);",
+     "        gamma[j] = (float)(1.0 / c[j]);"),
+    ("temporal_scale_qmax", "codec.c",
+     "            double s16 = or_fp16_round(clampd((float)((double)amax / qm), F16_MIN_NORMAL, F16_MAX));",
+     "            double s16 = or_fp16_round(clampd((float)((double)amax / (qm + 1)), F16_MIN_NORMAL, F16_MAX));"),
+    ("intb_scale_qmax", "codec.c", "        float s = (float)((double)amax / qm);",
+     "        float s = (float)((double)amax / (qm + 1));"),
+    ("fp16_ties_away", "numerics.c",
+     "    double n = nearbyint(a / quantum);    /* exact quotient; default mode is ties-to-even */",
+     "    double n = round(a / quantum);"),
+    ("lifetime_factor_two", "plan.c", "        L += exp(2.0 * j * ell);", "        L += exp(j * ell);"),
+    ("row_weight_exponent", "plan.c", "    const double half_gamma = 0.125;", "    const double half_gamma = 0.25;"),
+    ("dp_predecessor", "plan.c", "                double val = cost[(size_t)u * n_cand + k] + Fn[c - a];",
+     "                double val = cost[(size_t)u * n_cand + k] + Fn[c];"),
+    ("lagrangian_price", "plan.c", "            double val = cost[(size_t)u * n_cand + k] + lam * cands[k];",
+     "            double val = cost[(size_t)u * n_cand + k] + lam;"),
+    ("repair_slack_off_by_one", "plan.c", "                if (db <= 0 || db > slack)",
+     "                if (db <= 0 || db >= slack)"),
+    ("pivots_lowest_risk", "plan.c", "            if (!pivot[u] && (best < 0 || risk[u] > risk[best]))",
+     "            if (!pivot[u] && (best < 0 || risk[u] < risk[best]))"),
+    ("pivot_budget_16", "plan.c", "(long long)nominal * n_units - 8LL * n_piv",
+     "(long long)nominal * n_units - 16LL * n_piv"),
+    ("slot_stride_128", "plan.c", "    *slot_stride = (off + 255) / 256 * 256;",
+     "    *slot_stride = (off + 127) / 128 * 128;"),
+    ("gqa_interleaved", "batch.c", "    int hk = h / (Hv / Hk);\n    const float *g = gate_per_row ? gate + ((size_t)b * Hv + h) * OR_D : gate",
+     "    int hk = h % Hk;\n    const float *g = gate_per_row ? gate + ((size_t)b * Hv + h) * OR_D : gate"),
+    ("slot_ignored", "batch.c", "    return pool + (uint64_t)slots[b] * stride + head_off[h];",
+     "    return pool + (uint64_t)b * stride + head_off[h];"),
+]
+
+
+def _build(dst, edit=None):
+    os.makedirs(dst, exist_ok=True)
+    for f in SOURCES + ["oracle.h"]:
+        shutil.copy(os.path.join(ORACLE, f), dst)
+    if edit:
+        fname, old, new = edit
+        path = os.path.join(dst, fname)
+        src = open(path).read()
+        assert src.count(old) == 1, f"mutation site not unique in {fname}: {old!r}"
+        open(path, "w").write(src.replace(old, new))
+    so = os.path.join(dst, "liboracle.so")
+    subprocess.run(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
+                    "-o", so] + [os.path.join(dst, f) for f in SOURCES] + ["-lm"], check=True)
+    return so
+
+
+def _run_pins(so):
+    env = dict(os.environ, STEPQ_ORACLE_LIB=so, OMP_NUM_THREADS="2")
+    return subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                           "-m", "not gpu"] + PINS, cwd=ROOT, env=env, capture_output=True, text=True,
+                          timeout=900)
+
+
+def test_unmodified_copy_passes_the_pins(tmp_path):
+    r = _run_pins(_build(str(tmp_path / "control")))
+    assert r.returncode == 0, r.stdout[-3000:]
+
+
+@pytest.mark.parametrize("mid,fname,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_planted_mistake_fails_a_pin(tmp_path, mid, fname, old, new):
+    r = _run_pins(_build(str(tmp_path / mid), (fname, old, new)))
+    assert r.returncode == 1, f"{mid} passed every pin:\n{r.stdout[-3000:]}"

@@ -155,3 +155,66 @@ def test_kda_packed_bytes(oracle, rng, key):
     if "fp32_mib" in g:
         assert 4 * N == g["fp32_mib"] * 2 ** 20
     assert stride % 256 == 0 and stride >= total
+
+
+def _pick(cost, cands, lam):
+    """argmin_k cost[u][k] + lam cands[k] per unit, ties to the narrower code
+    (the relaxed problem of App. C.2, written out with numpy)."""
+    b = np.asarray(cands, np.float64)
+    order = np.argsort(b, kind="stable")
+    val = cost[:, order] + lam * b[order]
+    return order[np.argmin(val, axis=1)]
+
+
+@pytest.mark.parametrize("cands", [(4, 6, 8), (2, 4, 6, 8)])
+def test_lagrangian_multiplier_is_the_budget_threshold(oracle, rng, cands):
+    """The shared multiplier is the smallest lambda whose relaxed choices fit:
+    they fit at lambda, and just below it they do not (0 when everything fits)."""
+    c = np.asarray(cands)
+    for _ in range(40):
+        U = int(rng.integers(2, 9))
+        cost = _random_costs(rng, U, cands)
+        budget = int(rng.integers(min(cands) * U, max(cands) * U + 1))
+        lam = oracle.lagrangian_multiplier(cost, cands, budget)
+        assert lam is not None and lam >= 0.0
+        assert c[_pick(cost, cands, lam)].sum() <= budget
+        if lam > 0.0:
+            assert c[_pick(cost, cands, lam * (1 - 1e-9))].sum() > budget
+        else:
+            assert c[_pick(cost, cands, 0.0)].sum() <= budget
+    assert oracle.lagrangian_multiplier(np.ones((3, 3)), (4, 6, 8), 11) is None
+
+
+@pytest.mark.parametrize("cands", [(4, 6, 8), (2, 4, 6, 8)])
+def test_repair_leaves_no_fitting_upgrade(oracle, rng, cands):
+    """The discrete repair upgrades while an upgrade with non-negative gain still
+    fits the remaining budget; afterwards none does."""
+    for _ in range(40):
+        U = int(rng.integers(2, 9))
+        cost = _random_costs(rng, U, cands)
+        budget = int(rng.integers(min(cands) * U, max(cands) * U + 1))
+        ch = oracle.allocate_lagrangian(cost, cands, budget)
+        slack = budget - sum(cands[k] for k in ch)
+        assert slack >= 0
+        for u, cur in enumerate(ch):
+            for k, b in enumerate(cands):
+                db = b - cands[cur]
+                if 0 < db <= slack:
+                    assert cost[u, cur] - cost[u, k] < 0, (u, cur, k, slack)
+
+
+def test_layout_offsets_and_stride(oracle):
+    """Head segments follow one another in (layer, head) order, each as long as
+    its head page; the slot stride is their sum rounded up to 256 bytes. The row
+    widths make one head page 128 bytes past a multiple of 256."""
+    rb = np.full(D, 4, np.int8)
+    rb[:4] = 6                                      # sum of widths = 520 = 8 (mod 16)
+    rb2 = np.full(D, 8, np.int8)
+    bits = np.concatenate([rb, rb2, rb])
+    off, nb, stride = oracle.layout(ROW, 3, 1, bits)
+    sizes = [512 + 16 * int(r.astype(int).sum()) for r in (rb, rb2, rb)]
+    assert list(nb) == sizes
+    assert list(off) == [0, sizes[0], sizes[0] + sizes[1]]
+    assert sizes[0] % 256 == 128
+    assert stride % 256 == 0 and 0 <= stride - sum(sizes) < 256
+    assert oracle.layout(ROW, 1, 1, rb)[2] == 8960

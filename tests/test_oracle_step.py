@@ -123,3 +123,66 @@ def test_end_to_end_tiny_calibration_and_plan(oracle):
     assert plan.unit_bits.shape == (4,)
     assert np.sum(plan.unit_bits) <= 6 * 4
     assert plan.slot_stride == int(np.sum(plan.head_bytes))
+
+
+@pytest.mark.parametrize("bits,per_row", [(8, False), (6, True), (4, False)])
+def test_intb_step_is_recurrence_on_decoded_state(oracle, rng, bits, per_row):
+    """Uniform INT-b baseline step (App. B.5): the readout is the Delta update of
+    the decoded state (Eq. delta_update, fp64), and the new page is the rowwise
+    encoding of that updated tile."""
+    S = (rng.standard_normal((D, D)) * np.exp(rng.normal(size=(D, 1)))).astype(np.float32)
+    page = oracle.intb_encode_head(S, bits)
+    q, k, v, beta, gate = _inp(rng, per_row)
+    page1, y = oracle.intb_step_head(page, bits, q, k, v, beta, gate)
+    Shat = oracle.intb_decode_head(page, bits)
+    Dg = np.broadcast_to(gate.astype(np.float64), (D,))[:, None]
+    k64, v64, q64 = k.astype(np.float64), v.astype(np.float64), q.astype(np.float64)
+    P = Dg * Shat
+    X = P + float(beta) * np.outer(k64, v64 - k64 @ P)
+    yref = X.T @ q64
+    assert np.abs(y - yref).max() <= 2e-6 * np.abs(yref).max()
+    ref = oracle.intb_encode_head(X.astype(np.float32), bits)
+    assert np.array_equal(page1[:256], ref[:256])                     # row scales
+    assert np.mean(page1[256:] != ref[256:]) <= 1e-3                   # codes (fp32 rounding ties)
+
+
+def test_pool_step_is_the_per_unit_step(oracle, rng):
+    """The pool driver steps each (slot, value head) unit on its own page: value
+    head h reads key head h // (Hv / Hk) (grouped-query sharing), batch entry b
+    works on slot slots[b], and the other slots stay untouched."""
+    Hk, Hv, n_slots = 2, 4, 5
+    slots = np.array([3, 0, 4], np.int32)
+    B = len(slots)
+    cands = (4, 6, 8)
+    dist = np.sort(np.exp(rng.normal(0, 1, (Hv, 4))), axis=1)[:, ::-1].copy()
+    plan = oracle.make_plan(HEAD, 1, Hk, Hv, 6, cands, 1, 64, 1,
+                            np.exp(rng.normal(0, 1, (1, Hv, D))).astype(np.float32),
+                            rng.normal(-0.02, 0.01, Hv), dist)
+    pool = np.zeros(n_slots * plan.slot_stride, np.uint8)
+    states = rng.standard_normal((B, Hv, D, D)).astype(np.float32)
+    oracle.pool_encode(plan, pool, 0, slots, states)
+    before = pool.copy()
+
+    class Inp:
+        pass
+    inp = Inp()
+    inp.q = rng.standard_normal((B, Hk, D)).astype(np.float32)
+    inp.k = rng.standard_normal((B, Hk, D)).astype(np.float32)
+    inp.k /= np.linalg.norm(inp.k, axis=-1, keepdims=True)
+    inp.v = rng.standard_normal((B, Hv, D)).astype(np.float32)
+    inp.beta = rng.uniform(0.1, 0.9, (B, Hv)).astype(np.float32)
+    inp.gate = rng.uniform(0.9, 0.999, (B, Hv)).astype(np.float32)
+    y = oracle.pool_step(plan, pool, 0, slots, inp)
+    rb_layer, w_layer = plan.layer_row_bits(0), plan.layer_w(0)
+    for b in range(B):
+        for h in range(Hv):
+            o = int(slots[b]) * plan.slot_stride + int(plan.head_off[h])
+            n = int(plan.head_bytes[h])
+            page1, yu = oracle.step_head(before[o:o + n], HEAD, rb_layer[h], w_layer[h],
+                                         inp.q[b, h // 2], inp.k[b, h // 2], inp.v[b, h],
+                                         inp.beta[b, h], inp.gate[b, h])
+            assert np.array_equal(y[b, h], yu)
+            assert np.array_equal(pool[o:o + n], page1)
+    for s in set(range(n_slots)) - set(slots.tolist()):
+        seg = slice(s * plan.slot_stride, (s + 1) * plan.slot_stride)
+        assert np.array_equal(pool[seg], before[seg])
