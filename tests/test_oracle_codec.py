@@ -219,6 +219,31 @@ def test_column_update_minimises_weighted_error(oracle, rng, unit):
         assert abs(0.5 * (lo + hi) - c[j]) <= 1e-5 * c[j]
 
 
+@pytest.mark.parametrize("unit", [HEAD, ROW])
+def test_fit_starts_clip_free_and_takes_one_update(oracle, rng, unit):
+    """App. C.1: the column start is the smallest scale at which no integer row
+    clips, c0_j = max_i |X_ij| / (r_i zs_i qmax_i); one fixed-code update then
+    uses the nearest codes at c0 (clipped to +-qmax, which the start makes
+    unnecessary)."""
+    X = _state(rng)
+    rb = _widths(rng, unit, 6)
+    w = _w(rng)
+    nonpiv = rb != PIV
+    b = np.where(nonpiv, rb, 8).astype(np.float64)
+    zs = 2.0 ** (8 - b) if unit == ROW else np.ones(D)
+    qm = 2.0 ** (b - 1) - 1
+    r, c0, _ = oracle.fit_debug(X, unit, rb, w, 0)
+    Xd = X.astype(np.float64)
+    start = (np.abs(Xd[nonpiv]) / (r * zs * qm)[nonpiv, None]).max(axis=0)
+    assert np.allclose(c0, np.clip(start, 2.0 ** -14, 65504.0), rtol=1e-6)
+    r1, c1, z1 = oracle.fit_debug(X, unit, rb, w, 1)
+    assert np.array_equal(r1, r)
+    t = Xd[nonpiv] / (r * zs)[nonpiv, None] / c0.astype(np.float64)[None, :]
+    zref = np.clip(np.rint(t), -qm[nonpiv, None], qm[nonpiv, None])
+    assert np.mean(z1[nonpiv] != zref) <= 1e-4
+    assert np.all(np.abs(t) <= qm[nonpiv, None] * (1 + 1e-6))
+
+
 @pytest.mark.parametrize("bits", [4, 6, 8])
 def test_intb_baseline(oracle, rng, bits):
     """App. B.5: per key row s_i = fp16(absmax/q_b) in [2^-14, 65504], nearest codes."""

@@ -97,6 +97,45 @@ MUTANTS = [
      "    int hk = h % Hk;\n    const float *g = gate_per_row ? gate + ((size_t)b * Hv + h) * OR_D : gate"),
     ("slot_ignored", "batch.c", "    return pool + (uint64_t)slots[b] * stride + head_off[h];",
      "    return pool + (uint64_t)b * stride + head_off[h];"),
+    ("batch_recurrence_interleaved", "recurrence.c",
+     "            int hk = h / grp;\n            const float *g = gate_per_row ? gate + ((size_t)b * Hv + h) * OR_D\n"
+     "                                          : gate + (size_t)b * Hv + h;\n            or_delta_step_f32(",
+     "            int hk = h % Hk;\n            const float *g = gate_per_row ? gate + ((size_t)b * Hv + h) * OR_D\n"
+     "                                          : gate + (size_t)b * Hv + h;\n            or_delta_step_f32("),
+    ("omega_abs_not_square", "calib.c", "                omega_sum[(size_t)h * OR_D + i] += gi[i] * gi[i];",
+     "                omega_sum[(size_t)h * OR_D + i] += fabs(gi[i]);"),
+    ("logret_without_log", "calib.c", "                logret_sum[h] += log((double)g[0]);",
+     "                logret_sum[h] += (double)g[0];"),
+    ("logret_row_without_log", "calib.c", "                    logret_sum[(size_t)h * OR_D + i] += log((double)g[i]);",
+     "                    logret_sum[(size_t)h * OR_D + i] += (double)g[i];"),
+    ("distortion_head_unweighted", "calib.c",
+     "                        double w2 = (double)w[i] * (double)w[i], ei = 0.0;",
+     "                        double w2 = 1.0, ei = 0.0;"),
+    ("distortion_row_per_element_sum", "calib.c", "                        acc[((size_t)h * OR_D + i) * (n_cand + 1) + k] += ei / OR_D;",
+     "                        acc[((size_t)h * OR_D + i) * (n_cand + 1) + k] += ei;"),
+    ("row_codebook_spacing", "codec.c",
+     "static int zs_of(int unit_kind, int b) { return unit_kind == OR_UNIT_ROW ? 1 << (8 - b) : 1; }",
+     "static int zs_of(int unit_kind, int b) { return unit_kind == OR_UNIT_ROW ? 1 << (7 - b) : 1; }"),
+    ("zero_denominator_divides", "codec.c", "            if (den > 0.0)\n                c[j] =",
+     "            if (den >= 0.0)\n                c[j] ="),
+    ("row_scale_floor_zero", "codec.c", "        r[i] = or_fp16_round(clampd(t, F16_MIN_NORMAL, F16_MAX));",
+     "        r[i] = or_fp16_round(clampd(t, 0.0, F16_MAX));"),
+    ("extra_fit_iteration", "codec.c", "    for (int it = 0; it < fit_iters; it++) {\n        for (int j = 0; j < OR_D; j++) {\n            float gamma",
+     "    for (int it = 0; it <= fit_iters; it++) {\n        for (int j = 0; j < OR_D; j++) {\n            float gamma"),
+    ("pivot_rows_in_fit", "codec.c", "        in_fit[i] = (b != OR_PIVOT_BITS);", "        in_fit[i] = 1;"),
+    ("bits_msb_first", "codec.c", "        if ((u >> t) & 1u)\n            row[p >> 3] |=",
+     "        if ((u >> (b - 1 - t)) & 1u)\n            row[p >> 3] |="),
+    ("rows_stored_ascending", "codec.c", "        if (rb[t] > b || (rb[t] == b && t < i))",
+     "        if (rb[t] < b || (rb[t] == b && t < i))"),
+    ("band_of_row", "codec.c", "        size_t chunk = (size_t)(i / 16) * OR_D + (size_t)j;        /* band-major chunks */",
+     "        size_t chunk = (size_t)(i % 8) * OR_D + (size_t)j;        /* band-major chunks */"),
+    ("fp16_subnormal_scale", "numerics.c", "        return s | (uint16_t)(a / ldexp(1.0, -24));   /* subnormal: fraction counts 2^-24 */",
+     "        return s | (uint16_t)(a / ldexp(1.0, -23));   /* subnormal: fraction counts 2^-24 */"),
+    ("row_pivot_risk_without_fp16", "plan.c",
+     "            risk[u] = L[u] * (dist[(size_t)u * (n_cand + 1) + kn] -\n                              dist[(size_t)u * (n_cand + 1) + n_cand]);",
+     "            risk[u] = L[u] * (dist[(size_t)u * (n_cand + 1) + kn] -\n                              0.0 * dist[(size_t)u * (n_cand + 1) + n_cand]);"),
+    ("dp_ties_narrower", "plan.c", "            if (cands[order[b]] > cands[order[a]]) {",
+     "            if (cands[order[b]] < cands[order[a]]) {"),
 ]
 
 

@@ -103,14 +103,23 @@ def test_head_pivots_rank_residual_risk(oracle, rng):
     assert np.sum(bits[piv == 0]) + 8 * n_piv <= nominal * U
 
 
-def test_row_pivots_rank_fp16_reduction(oracle, rng):
+@pytest.mark.parametrize("fp16_share", [0.0, 0.95])
+def test_row_pivots_rank_fp16_reduction(oracle, rng, fp16_share):
+    """Row pivots go to the largest L_u (d_u(nominal) - d_u(FP16)); with the FP16
+    distortion a large share of d_u(nominal) the ranking differs from L d alone."""
     cands = (2, 4, 6, 8)
     U = 40
-    dist = np.concatenate([_random_costs(rng, U, cands), np.exp(rng.normal(-12, 1, (U, 1)))], axis=1)
+    d = _random_costs(rng, U, cands)
     L = np.exp(rng.normal(0, 1, U))
+    d16 = np.exp(rng.normal(-12, 1, U))
+    plain_top = np.argsort(-(L * d[:, 1]), kind="stable")[:5]
+    d16[plain_top] += fp16_share * d[plain_top, 1]      # FP16 barely helps these rows
+    dist = np.concatenate([d, d16[:, None]], axis=1)
     piv = oracle.select_pivots(ROW, cands, 4, L, dist, 5)
     risk = L * (dist[:, 1] - dist[:, 4])
     assert set(np.flatnonzero(piv)) == set(np.argsort(-risk, kind="stable")[:5])
+    if fp16_share > 0:
+        assert set(np.flatnonzero(piv)) != set(plain_top)
     bits = oracle.allocate(ROW, cands, 4, L, dist, piv)
     assert np.sum(bits[piv == 0]) + 8 * 5 <= 4 * U
 
@@ -218,3 +227,12 @@ def test_layout_offsets_and_stride(oracle):
     assert sizes[0] % 256 == 128
     assert stride % 256 == 0 and 0 <= stride - sum(sizes) < 256
     assert oracle.layout(ROW, 1, 1, rb)[2] == 8960
+
+
+def test_dp_keeps_the_wider_code_on_ties(oracle):
+    """The DP's tie rule (a reading; the paper fixes none): among choices of equal
+    cost it keeps the wider code, so equal costs with room for every unit at the
+    widest candidate give the widest."""
+    for cands in ((4, 6, 8), (2, 4, 6, 8)):
+        ch = oracle.allocate_dp(np.zeros((5, len(cands))), cands, max(cands) // 2 * 5)
+        assert all(cands[k] == max(cands) for k in ch)

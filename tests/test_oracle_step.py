@@ -83,21 +83,25 @@ def test_error_propagation_prop1(oracle, rng):
         assert np.abs((yq.astype(np.float64) - yr) - pred).max() <= 1e-4 * np.abs(yr).max()
 
 
-def test_calibration_omega_and_logret(oracle):
-    wl = W.WORKLOADS["gqa"].replace(batch=3)
+@pytest.mark.parametrize("name", ["gqa", "channel"])
+def test_calibration_omega_and_logret(oracle, name):
+    """omega sums g^2 with g = A^T q built densely; ell sums log alpha per head
+    (scalar gates) or log d_i per key channel (channel gates)."""
+    wl = W.WORKLOADS[name].replace(batch=3)
     mp = W.model_params(wl)
     inp = W.step_inputs(wl, mp, W.STREAM_CALIB, 0, 0, batch=3)
+    grp = wl.hv // wl.hk
     om = np.zeros((wl.hv, D))
-    lr = np.zeros(wl.hv)
+    lr = np.zeros((wl.hv, D) if wl.gate_per_row else wl.hv)
     oracle.calib_observe(inp, om, lr)
     for h in (0, 5, 31):
         ref = np.zeros(D)
         for b in range(3):
-            g = oracle.row_impact(inp.q[b, h // 2], inp.k[b, h // 2], inp.beta[b, h],
+            g = oracle.row_impact(inp.q[b, h // grp], inp.k[b, h // grp], inp.beta[b, h],
                                   inp.gate[b, h], dense=True)
             ref += g * g
         assert np.allclose(om[h], ref, rtol=1e-10)
-        assert np.isclose(lr[h], np.sum(np.log(inp.gate[:, h].astype(np.float64))))
+        assert np.allclose(lr[h], np.sum(np.log(inp.gate[:, h].astype(np.float64)), axis=0), rtol=1e-12)
 
 
 def test_calibration_distortion_driver(oracle, rng):
@@ -114,6 +118,27 @@ def test_calibration_distortion_driver(oracle, rng):
                 ref += np.sum(w[h][:, None].astype(np.float64) ** 2 * (R - S[s, h]) ** 2) / D / D
             assert np.isclose(acc[h, kk], ref, rtol=1e-12)
         assert acc[h, 0] > acc[h, 1] > acc[h, 2] > acc[h, 3] >= 0
+
+
+def test_calibration_distortion_driver_rows(oracle, rng):
+    """Row units (Eq. kda_calibration_distortion): per key row, the unweighted
+    mean squared error over its 128 elements, summed over the sampled states."""
+    S = (rng.standard_normal((2, 2, D, D)) * np.exp(rng.normal(size=(1, 1, D, 1)))).astype(np.float32)
+    w = np.exp(rng.normal(0, 0.3, (2, D))).astype(np.float32)
+    cands = (2, 4, 6, 8)
+    acc = np.zeros((2 * D, len(cands) + 1))
+    oracle.calib_distortion(ROW, S, w, cands, None, 1, acc)
+    for h in range(2):
+        for kk, b in enumerate(cands):
+            rb = np.full(D, b, np.int8)
+            ref = np.zeros(D)
+            for s in range(2):
+                R = oracle.decode_head(oracle.encode_head(S[s, h], ROW, rb, w[h]), ROW, rb)
+                ref += np.sum((R - S[s, h]) ** 2, axis=1) / D
+            assert np.allclose(acc[h * D:(h + 1) * D, kk], ref, rtol=1e-12)
+        f16 = sum(np.sum((np.float16(S[s, h]).astype(np.float64) - S[s, h]) ** 2, axis=1) / D
+                  for s in range(2))
+        assert np.allclose(acc[h * D:(h + 1) * D, len(cands)], f16, rtol=1e-12)
 
 
 def test_end_to_end_tiny_calibration_and_plan(oracle):
