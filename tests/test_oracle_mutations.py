@@ -139,19 +139,35 @@ MUTANTS = [
 ]
 
 
-def _build(dst, edit=None):
-    os.makedirs(dst, exist_ok=True)
+CFLAGS = ["-O2", "-std=c11", "-fPIC", "-fopenmp", "-ffp-contract=off"]
+
+
+@pytest.fixture(scope="module")
+def objects(tmp_path_factory):
+    """The unmodified sources compiled once; a mutant recompiles only its file."""
+    d = str(tmp_path_factory.mktemp("oracle_objs"))
     for f in SOURCES + ["oracle.h"]:
-        shutil.copy(os.path.join(ORACLE, f), dst)
+        shutil.copy(os.path.join(ORACLE, f), d)
+    for f in SOURCES:
+        subprocess.run(["gcc", "-c"] + CFLAGS + ["-o", os.path.join(d, f + ".o"), os.path.join(d, f)],
+                       check=True)
+    return d
+
+
+def _build(objs, dst, edit=None):
+    os.makedirs(dst, exist_ok=True)
+    parts = [os.path.join(objs, f + ".o") for f in SOURCES]
     if edit:
         fname, old, new = edit
-        path = os.path.join(dst, fname)
-        src = open(path).read()
+        src = open(os.path.join(objs, fname)).read()
         assert src.count(old) == 1, f"mutation site not unique in {fname}: {old!r}"
+        path = os.path.join(dst, fname)
         open(path, "w").write(src.replace(old, new))
+        obj = os.path.join(dst, fname + ".o")
+        subprocess.run(["gcc", "-c"] + CFLAGS + ["-I", objs, "-o", obj, path], check=True)
+        parts[SOURCES.index(fname)] = obj
     so = os.path.join(dst, "liboracle.so")
-    subprocess.run(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
-                    "-o", so] + [os.path.join(dst, f) for f in SOURCES] + ["-lm"], check=True)
+    subprocess.run(["gcc", "-shared", "-fopenmp", "-o", so] + parts + ["-lm"], check=True)
     return so
 
 
@@ -162,12 +178,12 @@ def _run_pins(so):
                           timeout=900)
 
 
-def test_unmodified_copy_passes_the_pins(tmp_path):
-    r = _run_pins(_build(str(tmp_path / "control")))
+def test_unmodified_copy_passes_the_pins(objects, tmp_path):
+    r = _run_pins(_build(objects, str(tmp_path / "control")))
     assert r.returncode == 0, r.stdout[-3000:]
 
 
 @pytest.mark.parametrize("mid,fname,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
-def test_planted_mistake_fails_a_pin(tmp_path, mid, fname, old, new):
-    r = _run_pins(_build(str(tmp_path / mid), (fname, old, new)))
+def test_planted_mistake_fails_a_pin(objects, tmp_path, mid, fname, old, new):
+    r = _run_pins(_build(objects, str(tmp_path / mid), (fname, old, new)))
     assert r.returncode == 1, f"{mid} passed every pin:\n{r.stdout[-3000:]}"
