@@ -579,7 +579,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     }
     // Step 2a: retrieval u_j = sum_i k_i a_i (c_j q_ij).
     {
-        uint64_t ua[4] = {0, 0, 0, 0}, ub[4] = {0, 0, 0, 0};
+        uint64_t ua[4] = {0, 0, 0, 0};              // one accumulator per column: fewer live registers
 #pragma unroll
         for (int p = 0; p < 4; p++) {
             uint64_t klo, khi;
@@ -587,11 +587,10 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
 #pragma unroll
             for (int c = 0; c < 4; c++) {
                 ua[c] = ffma2(klo, x2[2 * p][c], ua[c]);
-                ub[c] = ffma2(khi, x2[2 * p + 1][c], ub[c]);
+                ua[c] = ffma2(khi, x2[2 * p + 1][c], ua[c]);
             }
         }
-        const float v[1][4] = {{pair_sum(fadd2(ua[0], ub[0])), pair_sum(fadd2(ua[1], ub[1])),
-                                pair_sum(fadd2(ua[2], ub[2])), pair_sum(fadd2(ua[3], ub[3]))}};
+        const float v[1][4] = {{pair_sum(ua[0]), pair_sum(ua[1]), pair_sum(ua[2]), pair_sum(ua[3])}};
         cols_to_red<1>(t, S.red, 0, v);
     }
     if (__syncthreads_or(!ok)) return false;
@@ -609,7 +608,7 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     uint64_t dl[4];
 #pragma unroll
     for (int c = 0; c < 4; c++) dl[c] = col_pair(S.colD, t.col(c));
-    uint64_t ya[4] = {0, 0, 0, 0}, yb[4] = {0, 0, 0, 0};
+    uint64_t ya[4] = {0, 0, 0, 0};                  // one accumulator per column
     float rs[16];
 #pragma unroll
     for (int p = 0; p < 4; p++) {
@@ -621,15 +620,18 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
             x2[2 * p][c] = ffma2(blo, dl[c], x2[2 * p][c]);
             x2[2 * p + 1][c] = ffma2(bhi, dl[c], x2[2 * p + 1][c]);
             ya[c] = ffma2(qlo, x2[2 * p][c], ya[c]);
-            yb[c] = ffma2(qhi, x2[2 * p + 1][c], yb[c]);
+            ya[c] = ffma2(qhi, x2[2 * p + 1][c], ya[c]);
         }
-        if (MODE == kFused) {
+    }
+    const float yp[4] = {pair_sum(ya[0]), pair_sum(ya[1]), pair_sum(ya[2]), pair_sum(ya[3])};
+    // row sums of |Z| once the readout accumulators are reduced (fewer live registers)
+    if (MODE == kFused) {
+#pragma unroll
+        for (int p = 0; p < 4; p++) {
             abs_row_sums(x2[2 * p], rs[4 * p], rs[4 * p + 1]);
             abs_row_sums(x2[2 * p + 1], rs[4 * p + 2], rs[4 * p + 3]);
         }
     }
-    const float yp[4] = {pair_sum(fadd2(ya[0], yb[0])), pair_sum(fadd2(ya[1], yb[1])),
-                         pair_sum(fadd2(ya[2], yb[2])), pair_sum(fadd2(ya[3], yb[3]))};
     if (B == kPivot || MODE == kReadout) {
         const float v[1][4] = {{yp[0], yp[1], yp[2], yp[3]}};
         cols_to_red<1>(t, S.red, 2, v);
