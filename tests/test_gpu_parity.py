@@ -69,6 +69,7 @@ def test_quantize_dequantize_pool(torch, name, kw, batch):
     ("tiny", dict(fit_iters=3), 1, 8),
     ("gqa", dict(nominal_bits=4, candidates=(2, 4, 6, 8), n_pivots=2), 16, 4),  # 2-bit heads
     ("channel", dict(fit_iters=2), 16, 3),                                     # row units, two LS passes
+    ("gqa", dict(fit_iters=2), 16, 3),                                         # head units, two LS passes
 ])
 def test_decode_step_teacher_forced(torch, name, kw, batch, steps):
     """App. C.3 steps 1-7 against the oracle, step by step."""
