@@ -267,6 +267,8 @@ def main():
             dist.barrier()
         torch.cuda.synchronize(dev)
 
+    wall_s = {}                                        # host wall time of each timed region
+
     def timed(fn, steps, warmup, per_launch=False, name="timed"):
         for s in range(warmup):
             fn(s)
@@ -276,6 +278,7 @@ def main():
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda.nvtx.range_push(name)
         e0.record(stream)
+        w0 = time.perf_counter()
         for s in range(steps):
             if per_launch:
                 fn(s, evs[s])
@@ -284,6 +287,7 @@ def main():
         e1.record(stream)
         torch.cuda.nvtx.range_pop()
         barrier()
+        wall_s[name] = time.perf_counter() - w0
         total_ms = e0.elapsed_time(e1)
         launch_ms = None
         if per_launch:
@@ -313,7 +317,8 @@ def main():
                 "frac": achieved / peak, "traffic": traffic,
                 "peak_source": "measured" if "hbm_gbs" in peaks else "fallback",
                 "bytes_per_launch": statistics.mean(layer_bytes),
-                "avg_launch_us": avg_launch_s * 1e6}
+                "avg_launch_us": avg_launch_s * 1e6,
+                "median_launch_us": statistics.median(launch_ms) * 1e3}
 
     # ---- end to end through the public API with host buffers ----
     # Every step copies each layer's inputs from pinned host memory and reads
@@ -404,6 +409,7 @@ def main():
                        "parallelism": f"replicas x{world}"},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": L * args.steps, "clocks": clk, "baselines": baselines,
+            "wall_s": {k: round(v, 4) for k, v in wall_s.items()},
         }
         print(json.dumps(line), flush=True)
     if world > 1:
