@@ -15,8 +15,9 @@
  *  - GQA: value head h reads key head h / (n_value_heads / n_key_heads).
  *  - Device buffers are allocated and owned by the caller. Device calls are
  *    asynchronous on the given stream (NULL = legacy default stream), never
- *    synchronise and never allocate. Argument errors return before anything is
- *    launched. Slot ids found out of range by a kernel skip that unit and raise
+ *    synchronise and never allocate, so they can be captured in a CUDA graph
+ *    (on a capturing stream) and replayed. Argument errors return before
+ *    anything is launched. Slot ids found out of range by a kernel skip that unit and raise
  *    a sticky error readable with stepq_device_error().
  *  - Within one call slot ids must be distinct (two units writing one page race);
  *    stepq_validate_slots() checks a slot list on the device.
