@@ -326,13 +326,30 @@ def main():
     # layers ahead of / one behind the kernel that uses them (three device
     # input buffers, ordered by events), so they overlap the decode kernels;
     # the step ends when the last y has reached the host.
+    # a layer's five inputs travel as one packed buffer (one copy per layer);
+    # the library gets a view of each
+    shapes = [x.shape for x in inputs[0][0]]
+    sizes = [x.numel() for x in inputs[0][0]]
+    total = sum(sizes)
+
+    def views(flat):
+        out, o = [], 0
+        for shp, n in zip(shapes, sizes):
+            out.append(flat[o:o + n].view(shp))
+            o += n
+        return out
+
     h_in = []
     for layer in range(L):
-        h_in.append([x.cpu().pin_memory() for x in inputs[0][layer]])
+        flat = torch.empty(total, dtype=torch.float32).pin_memory()
+        for dst, src in zip(views(flat), inputs[0][layer]):
+            dst.copy_(src)
+        h_in.append(flat)
     n_buf = 3
-    d_in = [[torch.empty_like(x) for x in inputs[0][0]] for _ in range(n_buf)]
+    d_flat = [torch.empty(total, dtype=torch.float32, device=dev) for _ in range(n_buf)]
+    d_in = [views(f) for f in d_flat]
     h_y = torch.empty((L, B, Hv, 128), dtype=torch.float32).pin_memory()
-    h2d = sum(x.numel() * x.element_size() for row in h_in for x in row)
+    h2d = sum(x.numel() * x.element_size() for x in h_in)
     d2h = h_y.numel() * 4
     h2d_stream, d2h_stream = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
     buf_free = [torch.cuda.Event() for _ in range(n_buf)]
@@ -355,8 +372,7 @@ def main():
             nb = (s * L + layer) % n_buf
             h2d_stream.wait_event(buf_free[nb])         # the kernel that last read this buffer
             with torch.cuda.stream(h2d_stream):
-                for dst, src in zip(d_in[nb], h_in[layer]):
-                    dst.copy_(src, non_blocking=True)
+                d_flat[nb].copy_(h_in[layer], non_blocking=True)
                 copied[nb].record(h2d_stream)
             stream.wait_event(copied[nb])
             stream.wait_event(y_read[layer])            # last step's y of this layer is on the host
