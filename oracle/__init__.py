@@ -252,9 +252,10 @@ def unpack_head(page, unit_kind, rb):
 
 
 def fit_debug(X, unit_kind, rb, w, fit_iters=1):
-    """(r values, last fp32 column iterate, codes of the last fixed-code update)."""
+    """(r values, last column iterate (exact, before FP16 rounding), codes of the
+    last fixed-code update)."""
     r = np.zeros(D, np.float64)
-    c = np.zeros(D, np.float32)
+    c = np.zeros(D, np.float64)
     z = np.zeros((D, D), np.int8)
     lib().or_fit_debug(_p(_f32(X)), unit_kind, _p(_i8(rb)), _p(_f32(w)), fit_iters, _p(r), _p(c),
                        _p(z))

@@ -9,17 +9,20 @@
  * share one column vector. FP16 pivots store X directly (Sec. 3.2).
  *
  * Readings where the paper is silent (listed in the design notes):
- *  - r_i = fp16(clamp(sqrt(m_i) * w_i^(-1/2), 2^-14, 65504)), the FP16 clamp of
- *    the baseline's scale storage (App. B.5);
+ *  - r_i = fp16(clamp(m_i^(1/2) w_i^(-1/2), 2^-14, 65504)) with m_i the exact
+ *    mean of |X_ij| over the row, the FP16 clamp of the baseline's scale storage
+ *    (App. B.5);
  *  - the column fit starts from the clip-free value
- *    c0_j = max_{i in I} |X_ij| / (r_i zs_i qmax_i) (evaluated in fp32 as
- *    max_i fp32(fp32(|X_ij| rho_i) / qmax_i)), then applies `fit_iters`
+ *    c0_j = max_{i in I} |X_ij| / (r_i zs_i qmax_i), then applies `fit_iters`
  *    fixed-code updates c_j = sum w_i^2 v_ij X_ij / sum w_i^2 v_ij^2 (App. C.1),
  *    a zero denominator keeping the current iterate, floor 2^-14, cap 65504;
- *  - "round to the nearest level" is round-half-to-even of the exact product
- *    X'_ij * gamma_j of the fp32 row-normalised value X'_ij = fp32(X * rho_i)
- *    and gamma_j = fp32(1/c_j), rho_i = fp32(1/(r_i zs_i)): one rounding, as a
- *    fused multiply-add with 1.5 * 2^23 takes it in the GPU tile;
+ *    the iterate is kept exactly (fp64) and rounded once, to FP16, for storage;
+ *  - "quantize each scaled entry X_ij / (r_i c_j) to the nearest representable
+ *    level" (Sec. 4.3) is taken literally: the nearest integer, ties to even, of
+ *    the exact quotient X_ij / (r_i zs_i c_j), then the clip to +-qmax_i. The
+ *    paper fixes no precision for this decision, so the oracle takes it on the
+ *    exact value; a kernel that evaluates the quotient in fp32 disagrees only
+ *    where it lies within a few fp32 ulps of a half-integer;
  *  - codes are stored offset-binary u = q + 2^(b-1), LSB-first per row.
  *
  * Page layout of one head (all pieces 16-byte multiples):
@@ -55,9 +58,31 @@ static double clampd(double x, double lo, double hi) { return x < lo ? lo : (x >
 
 /* fp32 product of two fp32 values (exact in fp64, rounded once) */
 static float mul32(float a, float b) { return (float)((double)a * (double)b); }
-/* Nearest integer (ties to even) to the exact product of two fp32 values: the
- * product of two floats is exact in fp64, so there is a single rounding. */
-static double rne_prod(float a, float b) { return rint((double)a * (double)b); }
+
+/* Nearest integer, ties to even, of the exact quotient x / d (d > 0), x an fp32
+ * value and d a product of FP16 values and a power of two. The rounded fp64
+ * quotient gives a candidate n; the remainder e = x - n d is exact in fp64
+ * whenever |n| <= 2^8 (n d has at most 30 significant bits and lies within d/2
+ * of x), which covers every code that is not clipped, and it decides the two
+ * cases where the rounded quotient lands on the wrong side of a half-integer. */
+static double rne_div(double x, double d)
+{
+    double n = rint(x / d);
+    double e = x - n * d;
+    int odd = fmod(n, 2.0) != 0.0;
+    if (2.0 * e > d || (2.0 * e == d && odd))
+        n += 1.0;
+    else if (-2.0 * e > d || (-2.0 * e == d && odd))
+        n -= 1.0;
+    return n;
+}
+
+/* The level of X_ij at the row scale r_i zs_i and column scale c_j, clipped to
+ * +-qmax (Eq. uniform_quantization with the dual-axis scale of Sec. 4.3). */
+static double level(float x, double r_zs, double c, int qm)
+{
+    return clampd(rne_div((double)x, r_zs * c), -qm, qm);
+}
 
 size_t or_head_bytes(int unit_kind, const int8_t *rb)
 {
@@ -172,77 +197,69 @@ void or_decode_head_f32(const uint8_t *page, int unit_kind, const int8_t *rb, fl
 
 /* Key-Row-Aware Dual-axis Fitting of an updated tile X (fp32, row-major)
  * (Sec. 4.3; App. C.1; App. C.3 steps 4-5). Outputs the FP16 row factors r,
- * the per-row reciprocal rho_i = fp32(1/(r_i zs_i)), the final fp32 column
- * iterate and the codes of the last fixed-code update (for inspection). */
+ * the final column iterate c (exact, before its FP16 rounding) and the codes of
+ * the last fixed-code update (for inspection). */
 static void fit_head(const float *X, int unit_kind, const int8_t *rb, const float *w,
-                     int fit_iters, double *r, float *rho, float *c, int8_t *z_last)
+                     int fit_iters, double *r, double *c, int8_t *z_last)
 {
-    float mu[OR_D];           /* fp32(1 / qmax_i) */
     int in_fit[OR_D];         /* non-pivot integer rows: the set I */
+    double rz[OR_D];          /* r_i zs_i */
     for (int i = 0; i < OR_D; i++) {
         int b = rb[i];
         in_fit[i] = (b != OR_PIVOT_BITS);
         if (!in_fit[i]) {
-            r[i] = 0.0;
-            rho[i] = mu[i] = 0.0f;
+            r[i] = rz[i] = 0.0;
             continue;
         }
         /* Row factors: m_i = (1/d_v) sum_j |X_ij|, r_i = m_i^(1/2) w_i^(-1/2). */
         double s = 0.0;
         for (int j = 0; j < OR_D; j++)
             s += fabs((double)X[i * OR_D + j]);
-        float m = (float)(s / OR_D);
-        float wis = (float)(1.0 / sqrt((double)w[i]));
-        float t = mul32(sqrtf(m), wis);
+        double m = s / OR_D;
+        double t = sqrt(m) / sqrt((double)w[i]);
         r[i] = or_fp16_round(clampd(t, F16_MIN_NORMAL, F16_MAX));
-        double zs = zs_of(unit_kind, b);
-        rho[i] = (float)(1.0 / (r[i] * zs));
-        mu[i] = (float)(1.0 / qmax_of(b));
+        rz[i] = r[i] * (double)zs_of(unit_kind, b);
     }
-    /* Column factors: clip-free start c0_j = max_i |X_ij| / (r_i zs_i qmax_i),
-     * evaluated as max_i fp32(fp32(|X_ij| rho_i) mu_i), then fixed-code
-     * least-squares updates of min_c sum_ij w_i^2 (X_ij - r_i c_j z_ij)^2 over
-     * the rows in I. */
+    /* Column factors: clip-free start c0_j = max_{i in I} |X_ij| / (r_i zs_i qmax_i),
+     * then fixed-code least-squares updates of
+     * min_c sum_{i in I} w_i^2 (X_ij - r_i c_j z_ij)^2 (v_ij = r_i zs_i q_ij). */
     for (int j = 0; j < OR_D; j++) {
-        float cmax = 0.0f;
+        double cmax = 0.0;
         for (int i = 0; i < OR_D; i++)
             if (in_fit[i]) {
-                float a = mul32(mul32(fabsf(X[i * OR_D + j]), rho[i]), mu[i]);
+                double a = fabs((double)X[i * OR_D + j]) / (rz[i] * qmax_of(rb[i]));
                 if (a > cmax)
                     cmax = a;
             }
-        c[j] = (float)clampd(cmax, F16_MIN_NORMAL, F16_MAX);
+        c[j] = clampd(cmax, F16_MIN_NORMAL, F16_MAX);
     }
     if (z_last)
         for (int t = 0; t < OR_N; t++)
             z_last[t] = 0;
     for (int it = 0; it < fit_iters; it++) {
         for (int j = 0; j < OR_D; j++) {
-            float gamma = (float)(1.0 / (double)c[j]);
             double num = 0.0, den = 0.0;
             for (int i = 0; i < OR_D; i++) {
                 if (!in_fit[i])
                     continue;
-                int b = rb[i], qm = qmax_of(b);
-                double qv = clampd(rne_prod(mul32(X[i * OR_D + j], rho[i]), gamma), -qm, qm);
+                double qv = level(X[i * OR_D + j], rz[i], c[j], qmax_of(rb[i]));
                 if (z_last)
                     z_last[i * OR_D + j] = (int8_t)qv;
-                double v = r[i] * (double)zs_of(unit_kind, b) * qv;      /* v_ij = r_i z_ij */
+                double v = rz[i] * qv;                                    /* v_ij = r_i z_ij */
                 double w2 = (double)w[i] * (double)w[i];
                 num += w2 * v * (double)X[i * OR_D + j];
                 den += w2 * v * v;
             }
             if (den > 0.0)
-                c[j] = (float)clampd((double)(float)(num / den), F16_MIN_NORMAL, F16_MAX);
+                c[j] = clampd(num / den, F16_MIN_NORMAL, F16_MAX);
         }
     }
 }
 
 void or_fit_debug(const float *X, int unit_kind, const int8_t *rb, const float *w,
-                  int fit_iters, double *r, float *c_iter, int8_t *z_last)
+                  int fit_iters, double *r, double *c_iter, int8_t *z_last)
 {
-    float rho[OR_D];
-    fit_head(X, unit_kind, rb, w, fit_iters, r, rho, c_iter, z_last);
+    fit_head(X, unit_kind, rb, w, fit_iters, r, c_iter, z_last);
 }
 
 /* Fit, then pack with the stored FP16 scales (App. C.3 step 6). */
@@ -258,23 +275,18 @@ void or_encode_head(const float *X, int unit_kind, const int8_t *rb, const float
             }
         return;
     }
-    double r[OR_D];
-    float rho[OR_D], c[OR_D];
-    fit_head(X, unit_kind, rb, w, fit_iters, r, rho, c, NULL);
-    /* Storage precision and final codes with the stored scales. */
+    double r[OR_D], c[OR_D];
+    fit_head(X, unit_kind, rb, w, fit_iters, r, c, NULL);
+    /* Storage precision, then the final codes with the stored scales. */
     double c16[OR_D];
-    float gamma[OR_D];
-    for (int j = 0; j < OR_D; j++) {
+    for (int j = 0; j < OR_D; j++)
         c16[j] = or_fp16_round(c[j]);
-        gamma[j] = (float)(1.0 / c16[j]);
-    }
     for (int i = 0; i < OR_D; i++) {
         put_u16(page + 2 * i, or_fp16_encode(r[i]));
         put_u16(page + 256 + 2 * i, or_fp16_encode(c16[i]));
     }
     for (int i = 0; i < OR_D; i++) {
         int b = rb[i];
-        int qm = b == OR_PIVOT_BITS ? 0 : qmax_of(b);
         for (int j = 0; j < OR_D; j++) {
             int pos;
             uint8_t *stream = page + elem_stream(unit_kind, rb, i, j, &pos);
@@ -282,7 +294,8 @@ void or_encode_head(const float *X, int unit_kind, const int8_t *rb, const float
                 put_u16(stream + pos / 8, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
                 continue;
             }
-            int qv = (int)clampd(rne_prod(mul32(X[i * OR_D + j], rho[i]), gamma[j]), -qm, qm);
+            double rz = r[i] * (double)zs_of(unit_kind, b);
+            int qv = (int)level(X[i * OR_D + j], rz, c16[j], qmax_of(b));
             put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1))));
         }
     }

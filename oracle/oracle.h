@@ -72,7 +72,7 @@ void or_step_head(uint8_t *page, int unit_kind, const int8_t *row_bits, const fl
                   int fit_iters, const float *q, const float *k, const float *v,
                   float beta, const float *gate, int gate_per_row, float *y);
 void or_fit_debug(const float *X, int unit_kind, const int8_t *row_bits, const float *w,
-                  int fit_iters, double *r, float *c_iter, int8_t *z_last);
+                  int fit_iters, double *r, double *c_iter, int8_t *z_last);
 void or_unpack_head(const uint8_t *page, int unit_kind, const int8_t *row_bits,
                     uint16_t *r, uint16_t *c, int8_t *codes, uint16_t *piv);
 

@@ -304,3 +304,23 @@ def test_temporal_mixed_widths_and_pivots(oracle, rng):
             assert np.all(np.abs(R[i] - x) <= s[i] * (0.5 + 1e-5) + (np.abs(q) == qm) * np.abs(x))
         off += 16 * b
     assert off == page.size
+
+
+def test_code_ties_go_to_even(oracle):
+    """Sec. 4.3 quantizes X_ij / (r_i c_j) to the nearest level; an exact tie
+    (the quotient a half-integer) goes to the even level. Rows with mean |X| = 1
+    and w = 1 get r_i = 1, and a column whose largest entry is qmax = 127 gets
+    the clip-free start c0 = 1, so the first fixed-code pass quantizes X_i0
+    itself."""
+    X = np.zeros((D, D), np.float32)
+    X[0, 0], X[0, 1] = 127.0, 1.0
+    ties = [0.5, 1.5, 2.5, 3.5, -0.5, -1.5, -2.5, 126.5]
+    for i, x in enumerate(ties, start=1):
+        X[i, 0] = x
+        X[i, 1] = 128.0 - abs(x)                   # mean |X_i| = 1
+    rb = np.full(D, 8, np.int8)
+    r, c0, _ = oracle.fit_debug(X, HEAD, rb, np.ones(D, np.float32), 0)
+    assert np.all(r[:len(ties) + 1] == 1.0) and c0[0] == 1.0
+    _, _, z = oracle.fit_debug(X, HEAD, rb, np.ones(D, np.float32), 1)
+    assert z[0, 0] == 127
+    assert [int(z[i, 0]) for i in range(1, len(ties) + 1)] == [0, 2, 2, 4, 0, -2, -2, 126]

@@ -58,19 +58,23 @@ MUTANTS = [
     ("intb_step_delta_sign", "codec.c", INTB_W, INTB_W.replace("((double)v[j] - u[j])", "(u[j] - (double)v[j])")),
     ("ls_weight_w_not_w2", "codec.c", "                double w2 = (double)w[i] * (double)w[i];",
      "                double w2 = (double)w[i];"),
-    ("row_factor_exponent", "codec.c", "        float wis = (float)(1.0 / sqrt((double)w[i]));",
-     "        float wis = (float)sqrt((double)w[i]);"),
-    ("column_start_without_mu", "codec.c",
-     "                float a = mul32(mul32(fabsf(X[i * OR_D + j]), rho[i]), mu[i]);",
-     "                float a = mul32(fabsf(X[i * OR_D + j]), rho[i]);"),
-    ("codes_truncated", "codec.c",
-     "static double rne_prod(float a, float b) { return rint((double)a * (double)b); }",
-     "static double rne_prod(float a, float b) { return trunc((double)a * (double)b); }"),
+    ("row_factor_exponent", "codec.c", "        double t = sqrt(m) / sqrt((double)w[i]);",
+     "        double t = sqrt(m) * sqrt((double)w[i]);"),
+    ("column_start_without_qmax", "codec.c",
+     "                double a = fabs((double)X[i * OR_D + j]) / (rz[i] * qmax_of(rb[i]));",
+     "                double a = fabs((double)X[i * OR_D + j]) / rz[i];"),
+    ("codes_floored", "codec.c", "    return clampd(rne_div((double)x, r_zs * c), -qm, qm);",
+     "    return clampd(floor((double)x / (r_zs * c)), -qm, qm);"),
+    ("code_ties_up", "codec.c", "    if (2.0 * e > d || (2.0 * e == d && odd))",
+     "    if (2.0 * e > d || 2.0 * e == d)"),
+    ("code_clip_qmax_plus_one", "codec.c", "    return clampd(rne_div((double)x, r_zs * c), -qm, qm);",
+     "    return clampd(rne_div((double)x, r_zs * c), -qm - 1, qm + 1);"),
     ("offset_binary_bias", "codec.c",
      "            put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1))));",
      "            put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1)) - 1));"),
-    ("final_codes_unrounded_c", "codec.c", "        gamma[j] = (float)(1.0 / c16[j]);",
-     "        gamma[j] = (float)(1.0 / c[j]);"),
+    ("final_codes_unrounded_c", "codec.c",
+     "            int qv = (int)level(X[i * OR_D + j], rz, c16[j], qmax_of(b));",
+     "            int qv = (int)level(X[i * OR_D + j], rz, c[j], qmax_of(b));"),
     ("temporal_scale_qmax", "codec.c",
      "            double s16 = or_fp16_round(clampd((float)((double)amax / qm), F16_MIN_NORMAL, F16_MAX));",
      "            double s16 = or_fp16_round(clampd((float)((double)amax / (qm + 1)), F16_MIN_NORMAL, F16_MAX));"),
@@ -120,8 +124,8 @@ MUTANTS = [
      "            if (den >= 0.0)\n                c[j] ="),
     ("row_scale_floor_zero", "codec.c", "        r[i] = or_fp16_round(clampd(t, F16_MIN_NORMAL, F16_MAX));",
      "        r[i] = or_fp16_round(clampd(t, 0.0, F16_MAX));"),
-    ("extra_fit_iteration", "codec.c", "    for (int it = 0; it < fit_iters; it++) {\n        for (int j = 0; j < OR_D; j++) {\n            float gamma",
-     "    for (int it = 0; it <= fit_iters; it++) {\n        for (int j = 0; j < OR_D; j++) {\n            float gamma"),
+    ("extra_fit_iteration", "codec.c", "    for (int it = 0; it < fit_iters; it++) {\n        for (int j = 0; j < OR_D; j++) {\n            double num",
+     "    for (int it = 0; it <= fit_iters; it++) {\n        for (int j = 0; j < OR_D; j++) {\n            double num"),
     ("pivot_rows_in_fit", "codec.c", "        in_fit[i] = (b != OR_PIVOT_BITS);", "        in_fit[i] = 1;"),
     ("bits_msb_first", "codec.c", "        if ((u >> t) & 1u)\n            row[p >> 3] |=",
      "        if ((u >> (b - 1 - t)) & 1u)\n            row[p >> 3] |="),
