@@ -43,6 +43,20 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, long l
     return true;
 }
 
+// ---- small asynchronous copies (4 bytes, both addresses 4-byte aligned) ----
+// The per-item scalars (beta, a scalar gate) travel this way into the stage,
+// so that no thread waits on a global load when an item starts.
+__device__ __forceinline__ void cp_async4(void *dst_smem, const void *src_gmem) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(dst_smem)), "l"(src_gmem)
+                 : "memory");
+}
+// The current phase of `bar` also waits for this thread's earlier cp.async
+// copies: the pending arrival count goes up by one now and comes down when they
+// have landed. Issue it before the arrive that ends the thread's part of the phase.
+__device__ __forceinline__ void cp_async_mbar_arrive(uint64_t *bar) {
+    asm volatile("cp.async.mbarrier.arrive.shared::cta.b64 [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
 // ---- bulk (non-tensor) async copies: 16-byte aligned, size a multiple of 16 ----
 __device__ __forceinline__ void bulk_load(void *dst_smem, const void *src_gmem, uint32_t bytes,
                                           uint64_t *bar) {

@@ -27,7 +27,7 @@
 namespace stepq {
 namespace hk {
 
-constexpr int kVecBytes = 5 * 512;                     // q k v w2 wis per stage
+constexpr int kVecBytes = 5 * 512 + 128;               // q k v w2 wis | gate, beta per stage
 
 // ------------------------------------------------------------ shared layout
 constexpr int kOffBars = 0;                            // uint64 [8]
@@ -81,7 +81,7 @@ struct Smem {
 
 struct Stage {
     uint8_t *page;
-    float *q, *k, *v, *w2, *wis;
+    float *q, *k, *v, *w2, *wis, *gb;
     __device__ __forceinline__ Stage(uint8_t *base, uint32_t page_region) {
         page = base;
         q = (float *)(base + page_region);
@@ -89,6 +89,7 @@ struct Stage {
         v = q + 256;
         w2 = q + 384;
         wis = q + 512;
+        gb = q + 640;
     }
 };
 
@@ -504,7 +505,11 @@ __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h,
     Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
     const uint32_t nb = S.hbytes[h];
     const int hk = S.hkey[h];
-    constexpr uint32_t vec = MODE == kFused ? kVecBytes : 4 * 512 - (MODE == kReadout ? 512 : 0);
+    constexpr uint32_t vec = MODE == kFused ? 5 * 512 : 4 * 512 - (MODE == kReadout ? 512 : 0);
+    const size_t u = (size_t)b * a.Hv + h;
+    cp_async4(st.gb, a.gate + u);
+    cp_async4(st.gb + 1, a.beta + u);
+    cp_async_mbar_arrive(bar);
     mbar_arrive_tx(bar, nb + vec);
     bulk_load(st.page, a.pool + (uint64_t)slot * a.stride + S.hoff[h], nb, bar);
     if (MODE != kWriteback) bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
@@ -675,8 +680,8 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
         [&](int h, int b, int slot, int s) { issue<MODE>(a, S, h, b, slot, s); },
         [&](int h, int b, int, int s, bool ok, const auto &refill) {
             const size_t u = (size_t)b * a.Hv + h;
-            const float2 gb = make_float2(a.gate[u], a.beta[u]);
             const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
+            const float2 gb = *(const float2 *)st.gb;     // (gate, beta), staged with the page
             float *y_out = MODE == kWriteback ? nullptr : a.y + u * 128;
             float *d_out = MODE == kReadout ? a.delta + u * 128 : nullptr;
             switch (S.hbits[h]) {

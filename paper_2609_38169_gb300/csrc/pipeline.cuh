@@ -23,6 +23,36 @@ namespace pipe {
 
 constexpr long long kWaitCycles = 2000000000LL;      // ~1 s at 2 GHz
 constexpr int kProducer = kThreads - 32;              // lane 0 of the last warp issues copies
+constexpr int kMaxStages = 4;                         // bars[0..4) barriers, bars[4..8) slot ids
+
+// Repeated slot ids (two entries of one call writing one page race): every
+// unordered pair of batch entries is compared once across the whole grid --
+// entry i against entries i+1 .. i+floor(nb/2), cyclically -- and a repeated
+// valid id raises STEPQ_ERR_DUP_SLOT. The check keeps no state, so launches that
+// overlap on other streams or replay in a graph cannot disturb it. It costs about
+// nb^2 / 2 comparisons per launch, a few per thread for nb = 1024.
+__device__ __forceinline__ void check_repeats(const int32_t *slots, int nb, int pool_slots,
+                                              unsigned int *err) {
+    const long long half = nb / 2, pairs = (long long)nb * half;
+    const long long threads = (long long)gridDim.x * blockDim.x;
+    const long long chunk = (pairs + threads - 1) / threads;
+    long long p = ((long long)blockIdx.x * blockDim.x + threadIdx.x) * chunk;
+    const long long end = p + chunk < pairs ? p + chunk : pairs;
+    if (p >= end) return;
+    int i = (int)(p / half), d = (int)(p - (long long)i * half) + 1;
+    int si = slots[i];
+    for (; p < end; p++) {
+        const int j = i + d < nb ? i + d : i + d - nb;
+        if (slots[j] == si && si >= 0 && si < pool_slots) {
+            raise_error(err, STEPQ_ERR_DUP_SLOT);
+            return;
+        }
+        if (++d > half) {
+            d = 1;
+            si = slots[++i < nb ? i : 0];
+        }
+    }
+}
 
 // (head, batch entry) of item = head * nb + entry, stepped by the grid stride
 // G = gq * nb + gr without divisions.
@@ -47,7 +77,10 @@ struct Shape {
     unsigned int *err;
 };
 
-// Runs the item loop of this CTA (all threads call it; bars[0..S) initialised).
+// Runs the item loop of this CTA (all threads call it; bars[0..S) initialised,
+// S <= kMaxStages; the 16 bytes at bars + kMaxStages are free for the slot id of
+// each stage, which the producer writes when it starts the stage and every
+// thread reads once the stage's barrier has completed).
 //   issue(h, b, slot, s)      producer only: arrive with expect_tx on bars[s]
 //                             and start the item's copies into stage s
 //   process(h, b, slot, s, ok, refill) -> bool
@@ -57,7 +90,9 @@ struct Shape {
 //                             stalled
 //   store(h, slot, s)         producer only: write the final page back
 // An item whose slot id is out of range raises STEPQ_ERR_SLOT_RANGE; its stage
-// completes without data and nothing is written.
+// completes without data and nothing is written. A slot id repeated within the
+// launch raises STEPQ_ERR_DUP_SLOT (check_repeats); the pages of that slot are
+// then undefined.
 template <class Issue, class Process, class Store>
 __device__ __forceinline__ void run(const Shape &p, uint64_t *bars, Issue &&issue, Process &&process,
                                     Store &&store) {
@@ -66,7 +101,9 @@ __device__ __forceinline__ void run(const Shape &p, uint64_t *bars, Issue &&issu
     const int gq = G / p.nb, gr = G - gq * p.nb;
     const int first = blockIdx.x;
     const auto slot_ok = [&](int slot) { return slot >= 0 && slot < p.pool_slots; };
+    volatile int *stage_slot = (volatile int *)(bars + kMaxStages);
     const auto start = [&](int h, int b, int slot, int s) {
+        stage_slot[s] = slot;                          // released by the arrive below
         if (slot_ok(slot)) issue(h, b, slot, s);
         else mbar_arrive(&bars[s]);
     };
@@ -80,22 +117,24 @@ __device__ __forceinline__ void run(const Shape &p, uint64_t *bars, Issue &&issu
             c0.step(G, gq, gr, p.nb);
         }
     }
+    check_repeats(p.slots, p.nb, p.pool_slots, p.err);
+    __syncthreads();                      // the first stages' slot ids are visible to every thread
     // iteration n >= lag refills stage (n - lag) mod S with item n - lag + S
     Cursor cur(first, p.nb), iss(first + S_n * G, p.nb);
-    int slot = p.slots[cur.b];
     int s = 0, is = 0;                    // stage of the current item, stage refilled next
     uint32_t parity = 0;
     for (int n = 0; cur.item < p.items; n++) {
-        // prefetch: the next item's slot (all threads) and the slot of the item
-        // this iteration will issue (producer)
         Cursor nxt = cur;
         nxt.step(G, gq, gr, p.nb);
-        const int nslot = nxt.item < p.items ? p.slots[nxt.b] : -1;
+        // prefetch: the slot of the item this iteration will issue (producer)
         const bool do_issue = n >= lag && iss.item < p.items;
         int islot = -1;
         if (tid == kProducer && do_issue) islot = p.slots[iss.b];
 
         const bool ok = mbar_wait(&bars[s], parity, kWaitCycles);
+        // the item's slot id: the producer wrote it when it started the stage,
+        // before at least one CTA barrier
+        const int slot = stage_slot[s];
         const bool valid = slot_ok(slot);
         if (!valid && tid == 0) raise_error(p.err, STEPQ_ERR_SLOT_RANGE);
         // Refill the stage of an earlier item (its store was committed `lag`
@@ -136,7 +175,6 @@ __device__ __forceinline__ void run(const Shape &p, uint64_t *bars, Issue &&issu
             bulk_commit();
         }
         cur = nxt;
-        slot = nslot;
         if (n >= lag) {
             iss.step(G, gq, gr, p.nb);
             if (++is == S_n) is = 0;

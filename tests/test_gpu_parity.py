@@ -280,3 +280,48 @@ def test_empty_batch_and_bad_slots(torch):
     assert int(status.item()) == 3
     A.stepq_validate_slots(torch.tensor([3, 1], dtype=torch.int32, device="cuda"), 4, scratch, status)
     assert int(status.item()) == 0
+
+
+@pytest.mark.parametrize("kind", ["heads", "heads_readout", "heads_writeback", "rows", "fp32", "int8"])
+@pytest.mark.parametrize("slots_list", [[1, 3, 1], [5, 0, 2, 4, 6, 7, 9, 5]])
+def test_repeated_slots_are_reported(torch, kind, slots_list):
+    """A slot id repeated within one call (two units writing one page) raises
+    STEPQ_ERR_DUP_SLOT on the device; a call with distinct ids raises nothing.
+    The second list repeats its first entry at the last position (the pair
+    enumeration's wrap-around)."""
+    wl = W.WORKLOADS["channel" if kind == "rows" else "tiny"].replace(pool_slots=16)
+    cfg, plan, oplan, _ = plans(wl)
+    B = len(slots_list)
+    hk, hv = wl.hk, wl.hv
+    gshape = (B, hv, 128) if wl.gate_per_row else (B, hv)
+    q = torch.randn((B, hk, 128), device="cuda")
+    k = torch.nn.functional.normalize(torch.randn((B, hk, 128), device="cuda"), dim=-1)
+    v = torch.randn((B, hv, 128), device="cuda")
+    beta = torch.full((B, hv), 0.5, device="cuda")
+    gate = torch.full(gshape, 0.95, device="cuda")
+    y = torch.empty((B, hv, 128), device="cuda")
+    delta = torch.zeros((B, hv, 128), device="cuda")
+    if kind == "fp32":
+        pool = torch.zeros((wl.pool_slots, wl.layers, hv, 128, 128), device="cuda")
+    elif kind == "int8":
+        pool = torch.zeros(wl.pool_slots * A.stepq_intb_slot_bytes(cfg, 8), dtype=torch.uint8, device="cuda")
+    else:
+        pool = A.alloc_pool(plan, wl.pool_slots)
+
+    def call(sl):
+        s_d = torch.tensor(sl, dtype=torch.int32, device="cuda")
+        if kind in ("heads", "rows"):
+            A.stepq_decode_step(plan, 0, pool, s_d, q, k, v, beta, gate, y)
+        elif kind == "heads_readout":
+            A.stepq_decode_readout(plan, 0, pool, s_d, q, k, v, beta, gate, y, delta)
+        elif kind == "heads_writeback":
+            A.stepq_decode_writeback(plan, 0, pool, s_d, k, beta, gate, delta)
+        elif kind == "fp32":
+            A.stepq_fp32_decode_step(cfg, 0, pool, s_d, q, k, v, beta, gate, y)
+        else:
+            A.stepq_intb_decode_step(cfg, 8, 0, pool, s_d, q, k, v, beta, gate, y)
+
+    call(slots_list)
+    assert A.stepq_device_error() == 3                                          # STEPQ_ERR_DUP_SLOT
+    call(list(range(B)))
+    assert A.stepq_device_error() == 0
