@@ -293,6 +293,41 @@ stepq_status stepq_calib_distortion(const stepq_config *cfg, int layer, const fl
                                     const uint8_t *pivot_rows, const float *states, int n,
                                     double *acc, stepq_stream_t stream);
 
+/* The whole calibration protocol of App. A.3 on a recorded trace, behind one
+ * call (the sequence of stepq_calib_observe, FP32-state replay and
+ * stepq_calib_distortion launches, the means and the pivot choice):
+ *   pass A  omega_i = mean_t g_{t,i}^2 (Sec. 4.1) and ell_u = mean_t log r_{t,u}
+ *           (Eq. calibration_lifetime) over the n * T tokens of every layer;
+ *   pass B  per layer, the FP32-state recurrence replayed from a zero state over
+ *           the T tokens of each sequence; every `every`-th state is fitted at
+ *           each candidate width (Eqs. qwen_calibration_distortion,
+ *           kda_calibration_distortion), one sample per sequence, and
+ *           d_u(b) is the mean over the samples;
+ *   pivots  as stepq_select_pivots from ell and the pass-B distortions; row
+ *           units then repeat pass B with the chosen pivot rows kept in FP16 and
+ *           out of the column fit (App. C.2), and that second measurement is
+ *           the `distortion` the plan takes.
+ * Trace, device fp32 (16-byte aligned; beta 4-byte): q, k [L][T][n][Hk][128];
+ * v [L][T][n][Hv][128]; beta [L][T][n][Hv]; gate [L][T][n][Hv] (scalar) or
+ * [L][T][n][Hv][128] (channel). workspace: device, 256-byte aligned, at least
+ * stepq_calib_workspace_bytes(cfg, n) bytes (contents clobbered). The result
+ * arrays are host memory the caller owns, written before the call returns.
+ * This is an offline call: it synchronises `stream` and allocates nothing. */
+typedef struct {
+    float *omega;               /* out [L][Hv][128] */
+    double *mean_log_ret;       /* out [units] */
+    double *distortion;         /* out [units][n_candidates+1], last column FP16 */
+    double *distortion_stage1;  /* out [units][n_candidates+1] of the first pass, or NULL */
+    uint8_t *pivot_mask;        /* out [units] */
+    int n_tokens, n_samples;    /* out: tokens per layer (n T) and samples per layer */
+} stepq_calib_result;
+size_t stepq_calib_workspace_bytes(const stepq_config *cfg, int n);
+stepq_status stepq_calibrate_from_trace(const stepq_config *cfg, int n, int T, int every,
+                                        const float *q, const float *k, const float *v,
+                                        const float *beta, const float *gate, void *workspace,
+                                        size_t workspace_bytes, stepq_calib_result *out,
+                                        stepq_stream_t stream);
+
 /* ----------------------------------------------------------------- diagnostics */
 /* Check on the device that slots[0..B) are distinct and in [0, pool_slots).
  * scratch: device, >= (pool_slots + 31) / 32 uint32 words (contents clobbered).
@@ -318,10 +353,22 @@ stepq_status stepq_validate_slots_noalloc(const int32_t *slots, int B, int pool_
 /* Read and clear the sticky device error of the current device (synchronises
  * `stream`): STEPQ_OK, or the first error a kernel raised. */
 stepq_status stepq_device_error(stepq_stream_t stream);
-/* The same read-and-clear of the sticky device error, under the name used for
- * it in the boundary's design table: surfaces what the asynchronous calls queued
- * on `stream` reported. Synchronises `stream`. */
+/* The same read-and-clear of the sticky device error under a second name:
+ * surfaces what the asynchronous calls queued on `stream` reported.
+ * Synchronises `stream`. */
 stepq_status stepq_stream_status(stepq_stream_t stream);
+
+/* Test support for the bounded waits (not for production use). Every wait of
+ * the pipelined decode kernels (stepq_decode_step, the split halves, the FP32
+ * and INT-b decode steps) gives up after `wait_cycles` SM clock cycles
+ * (default 2e9, about one second; at least 1000), raises STEPQ_ERR_TIMEOUT and
+ * lets its CTA return. withhold_item >= 0 makes every later launch skip the
+ * copies of that item (head * B + batch entry), so that its wait runs out and
+ * the launch reports STEPQ_ERR_TIMEOUT with its results undefined; -1 restores
+ * normal operation. The values are process-wide, read at each launch, and not
+ * safe to change while another thread launches. STEPQ_ERR_ARG for values out of
+ * range. The paper has no counterpart; this exists to test failure detection. */
+stepq_status stepq_debug_stall(long long wait_cycles, int withhold_item);
 
 const char *stepq_status_str(stepq_status s);
 const char *stepq_version(void);

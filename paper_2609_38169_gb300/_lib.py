@@ -21,6 +21,11 @@ class StepqCalib(C.Structure):
     _fields_ = [("omega", P), ("mean_log_ret", P), ("distortion", P), ("pivot_mask", P)]
 
 
+class StepqCalibResult(C.Structure):
+    _fields_ = [("omega", P), ("mean_log_ret", P), ("distortion", P), ("distortion_stage1", P),
+                ("pivot_mask", P), ("n_tokens", I), ("n_samples", I)]
+
+
 class StepqPlanInfo(C.Structure):
     _fields_ = [("slot_stride", SZ), ("n_units", SZ), ("unit_bits", P), ("pivot_mask", P),
                 ("w", P), ("lifetime", P), ("head_offset", P), ("head_bytes", P)]
@@ -54,6 +59,9 @@ SIGNATURES = {
     "stepq_intb_decode_step": (I, [CFG, I, I, P, I, P, I, P, P, P, P, P, P, P]),
     "stepq_calib_observe": (I, [CFG, I, P, P, P, P, I, P, P, P]),
     "stepq_calib_distortion": (I, [CFG, I, P, P, P, I, P, P]),
+    "stepq_calib_workspace_bytes": (SZ, [CFG, I]),
+    "stepq_debug_stall": (I, [C.c_longlong, I]),
+    "stepq_calibrate_from_trace": (I, [CFG, I, I, I, P, P, P, P, P, P, SZ, C.POINTER(StepqCalibResult), P]),
     "stepq_validate_slots": (I, [P, I, I, P, P, P]),
     "stepq_validate_slots_noalloc": (I, [P, I, I, P, P]),
     "stepq_device_error": (I, [P]),

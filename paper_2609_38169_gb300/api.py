@@ -390,6 +390,13 @@ def stepq_validate_slots_noalloc(slots, pool_slots: int, status_out, stream=None
           "stepq_validate_slots_noalloc")
 
 
+def stepq_debug_stall(wait_cycles: int = 2_000_000_000, withhold_item: int = -1):
+    """Test support: the wait bound of the pipelined decode kernels and an item
+    whose copies never start (stepq_debug_stall; -1 = none). Defaults restore
+    normal operation."""
+    check(_lib.lib().stepq_debug_stall(int(wait_cycles), int(withhold_item)), "stepq_debug_stall")
+
+
 def stepq_device_error(stream=None) -> int:
     return int(_lib.lib().stepq_device_error(_stream(stream)))
 
@@ -411,26 +418,50 @@ class CalibStats:
     extra: dict = field(default_factory=dict)
 
 
+def stepq_calibrate_from_trace(cfg: Config, q, k, v, beta, gate, every: int, stream=None) -> CalibStats:
+    """The calibration protocol of App. A.3 on a device trace (q, k [L][T][n][Hk][128],
+    v [L][T][n][Hv][128], beta [L][T][n][Hv], gate [L][T][n][Hv] or [L][T][n][Hv][128]),
+    all in the library (stepq_calibrate_from_trace); the workspace comes from torch."""
+    import torch
+    f = torch.float32
+    L, T, n = q.shape[0], q.shape[1], q.shape[2]
+    c = cfg.c()
+    lib = _lib.lib()
+    nbytes = lib.stepq_calib_workspace_bytes(C.byref(c), n)
+    if nbytes == 0:
+        raise ValueError("invalid configuration or sequence count")
+    ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=q.device)
+    base = (ws.data_ptr() + 255) // 256 * 256
+    U = stepq_num_units(cfg)
+    K1 = len(cfg.candidates) + 1
+    omega = np.zeros((cfg.n_layers, cfg.n_value_heads, D), np.float32)
+    ell = np.zeros(U, np.float64)
+    dist = np.zeros((U, K1), np.float64)
+    dist1 = np.zeros((U, K1), np.float64)
+    pivot = np.zeros(U, np.uint8)
+    res = _lib.StepqCalibResult(omega.ctypes.data, ell.ctypes.data, dist.ctypes.data, dist1.ctypes.data,
+                                pivot.ctypes.data, 0, 0)
+    check(lib.stepq_calibrate_from_trace(C.byref(c), n, T, int(every), _dev_ptr(q, f), _dev_ptr(k, f),
+                                         _dev_ptr(v, f), _dev_ptr(beta, f), _dev_ptr(gate, f),
+                                         C.c_void_p(base), nbytes, C.byref(res), _stream(stream)),
+          "stepq_calibrate_from_trace")
+    return CalibStats(omega, ell, dist1, dist, pivot, res.n_tokens, res.n_samples)
+
+
 def calibrate(cfg: Config, wl, device="cuda", seqs=None, steps=None, every=None,
               device_inputs: bool = False) -> CalibStats:
-    """Calibration statistics for `cfg` on the workload's calibration stream, all
-    arithmetic in the library's kernels (App. A.3): pass A accumulates omega and
-    ell; pass B replays the FP32-state recurrence from zero per layer and fits
-    sampled states at every candidate width; row units then fix their pivots and
-    repeat pass B with those rows held out of the column fit. `device_inputs`
-    draws the calibration stream on the GPU (fast, for full-size runs) instead of
-    with the numpy generator the oracle shares."""
+    """Calibration statistics for `cfg` on the workload's calibration stream
+    (App. A.3): the trace of `steps` tokens for `seqs` sequences per layer is
+    drawn (on the GPU with `device_inputs`, else with the numpy generator the
+    oracle shares) and handed to stepq_calibrate_from_trace, which does every
+    step of the protocol."""
     import torch
     from . import workloads as W
     seqs = wl.calib_seqs if seqs is None else seqs
     steps = wl.calib_steps if steps is None else steps
     every = wl.calib_every if every is None else every
     mp = W.model_params(wl)
-    L, Hv = cfg.n_layers, cfg.n_value_heads
-    n_units = stepq_num_units(cfg)
-    K1 = len(cfg.candidates) + 1
     dev = torch.device(device)
-
     mp_dev = W.model_params_torch(mp, dev) if device_inputs else None
 
     def inputs(t, layer):
@@ -439,38 +470,13 @@ def calibrate(cfg: Config, wl, device="cuda", seqs=None, steps=None, every=None,
         inp = W.step_inputs(wl, mp, W.STREAM_CALIB, t, layer, batch=seqs)
         return [torch.from_numpy(a).to(dev) for a in (inp.q, inp.k, inp.v, inp.beta, inp.gate)]
 
-    omega_sum = torch.zeros((L, Hv, D), dtype=torch.float64, device=dev)
-    logret_sum = torch.zeros(n_units, dtype=torch.float64, device=dev)
-    for t in range(steps):
-        for layer in range(L):
-            q, k, _, beta, gate = inputs(t, layer)
-            stepq_calib_observe(cfg, layer, q, k, beta, gate, omega_sum, logret_sum)
-    n_tok = seqs * steps
-    omega = (omega_sum / n_tok).float().cpu().numpy()
-    mean_log_ret = (logret_sum / n_tok).cpu().numpy()
-    w_dev = torch.from_numpy(stepq_row_weights(cfg, omega)).to(dev)
-    cfg1 = Config(**{**cfg.__dict__, "n_layers": 1})
-    slots = torch.arange(seqs, dtype=torch.int32, device=dev)
-
-    def distortion_pass(pivot_rows):
-        acc = torch.zeros((n_units, K1), dtype=torch.float64, device=dev)
-        n_samp = 0
-        for layer in range(L):
-            S = torch.zeros((seqs, Hv, D, D), dtype=torch.float32, device=dev)
-            y = torch.empty((seqs, Hv, D), dtype=torch.float32, device=dev)
-            for t in range(steps):
-                q, k, v, beta, gate = inputs(t, layer)
-                stepq_fp32_decode_step(cfg1, 0, S, slots, q, k, v, beta, gate, y)
-                if (t + 1) % every == 0:
-                    stepq_calib_distortion(cfg, layer, w_dev, pivot_rows, S, acc)
-                    if layer == 0:
-                        n_samp += seqs
-        return (acc / max(n_samp, 1)).cpu().numpy(), n_samp
-
-    d1, n_samp = distortion_pass(None)
-    pivot = stepq_select_pivots(cfg, mean_log_ret, d1)
-    if cfg.unit_rows and pivot.any():
-        d2, _ = distortion_pass(torch.from_numpy(pivot).to(dev))
-    else:
-        d2 = d1
-    return CalibStats(omega, mean_log_ret, d1, d2, pivot, n_tok, n_samp)
+    trace = None
+    for layer in range(cfg.n_layers):
+        for t in range(steps):
+            xs = inputs(t, layer)
+            if trace is None:
+                trace = [torch.empty((cfg.n_layers, steps) + tuple(x.shape), dtype=torch.float32, device=dev)
+                         for x in xs]
+            for dst, x in zip(trace, xs):
+                dst[layer, t].copy_(x)
+    return stepq_calibrate_from_trace(cfg, *trace, every=every)

@@ -13,7 +13,7 @@ BUILD = os.path.join(PKG, "_build")
 SO = os.path.join(BUILD, "libstepq.so")
 INCLUDE = os.path.join(ROOT, "include")
 SOURCES = ["plan.cpp", "api.cpp", "errors.cu", "stepq_kernels.cu", "heads.cu", "rows.cu", "baselines.cu", "intb.cu", "temporal.cu", "fp32.cu", "prefill.cu",
-           "calib.cu"]
+           "calib.cu", "calibrate.cu"]
 HEADERS = ["internal.h", "device.cuh", "async.cuh", "pipeline.cuh", "tile.cuh", "tcgen05.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -342,3 +342,7 @@ extern "C" const char *stepq_status_str(stepq_status s) {
 }
 
 extern "C" const char *stepq_version(void) { return "stepq 0.1 (sm_103a)"; }
+
+extern "C" stepq_status stepq_debug_stall(long long wait_cycles, int withhold_item) {
+    return set_stall_knob(wait_cycles, withhold_item);
+}

@@ -50,6 +50,17 @@ __device__ __forceinline__ void cp_async4(void *dst_smem, const void *src_gmem) 
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(dst_smem)), "l"(src_gmem)
                  : "memory");
 }
+// 16 bytes, both addresses 16-byte aligned (L2 only).
+__device__ __forceinline__ void cp_async16(void *dst_smem, const void *src_gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst_smem)), "l"(src_gmem)
+                 : "memory");
+}
+// A 512-byte vector copied by the 32 lanes of a warp, 16 bytes each: one
+// instruction for the warp, where a bulk copy would hold its issuing thread for
+// about a hundred cycles.
+__device__ __forceinline__ void warp_copy512(void *dst_smem, const void *src_gmem, int lane) {
+    cp_async16((uint8_t *)dst_smem + 16 * lane, (const uint8_t *)src_gmem + 16 * lane);
+}
 // The current phase of `bar` also waits for this thread's earlier cp.async
 // copies: the pending arrival count goes up by one now and comes down when they
 // have landed. Issue it before the arrive that ends the thread's part of the phase.

@@ -3,23 +3,49 @@
 // Kernels never trap: a unit whose slot id is out of range is skipped and the
 // first such status is latched in a per-device word that stepq_device_error()
 // reads and clears.
+#include <atomic>
+
 #include "device.cuh"
 #include "internal.h"
+#include "pipeline.cuh"
 
 namespace stepq {
 
+constexpr int kMaxDevices = 64;
+
 __device__ unsigned int g_error_word;
 
-unsigned int *device_error_word() {
-    static unsigned int *addr[64];
+// Device address of a file-scope __device__ variable on the current device,
+// looked up once per device. The cache entries are atomics: host threads that
+// make their first call on a device at the same time store the same address.
+static void *symbol_address(const void *symbol, std::atomic<void *> (&cache)[kMaxDevices]) {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    if (!addr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
-        addr[dev] = (unsigned int *)p;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    void *p = cache[dev].load(std::memory_order_acquire);
+    if (!p) {
+        if (cudaGetSymbolAddress(&p, symbol) != cudaSuccess || !p) return nullptr;
+        cache[dev].store(p, std::memory_order_release);
     }
-    return addr[dev];
+    return p;
+}
+
+unsigned int *device_error_word() {
+    static std::atomic<void *> addr[kMaxDevices];
+    return (unsigned int *)symbol_address((const void *)&g_error_word, addr);
+}
+
+// The pipelined kernels' wait bound and withheld item (test support). Plain
+// process-wide values: stepq_debug_stall is documented as not thread-safe.
+static long long g_wait_cycles = pipe::kWaitCycles;
+static int g_withhold_item = -1;
+
+StallKnob stall_knob() { return {g_wait_cycles, g_withhold_item}; }
+
+stepq_status set_stall_knob(long long wait_cycles, int withhold_item) {
+    if (wait_cycles < 1000 || withhold_item < -1) return STEPQ_ERR_ARG;
+    g_wait_cycles = wait_cycles;
+    g_withhold_item = withhold_item;
+    return STEPQ_OK;
 }
 
 stepq_status read_device_error(cudaStream_t s) {
@@ -67,21 +93,10 @@ static __device__ __align__(256) uint32_t g_slot_bitmap[kStaticSlotMax / 32];
 // Host code must not hand the symbol itself to a kernel: on the host it only
 // names a stand-in, not device memory.
 static uint32_t *static_bitmap(stepq_status *st) {
-    static uint32_t *addr[64];
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
-        *st = STEPQ_ERR_CUDA;
-        return nullptr;
-    }
-    if (!addr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_slot_bitmap) != cudaSuccess || !p) {
-            *st = STEPQ_ERR_CUDA;
-            return nullptr;
-        }
-        addr[dev] = (uint32_t *)p;
-    }
-    return addr[dev];
+    static std::atomic<void *> addr[kMaxDevices];
+    auto *p = (uint32_t *)symbol_address((const void *)g_slot_bitmap, addr);
+    if (!p) *st = STEPQ_ERR_CUDA;
+    return p;
 }
 
 stepq_status launch_validate_slots_static(const int32_t *slots, int B, int pool_slots,

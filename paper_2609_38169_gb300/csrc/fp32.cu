@@ -17,7 +17,7 @@ namespace stepq {
 namespace fk {
 
 constexpr int kPage = kN * 4;                          // 65,536 B
-constexpr int kVecBytes = 4 * 512;                     // q k v | gate (channel gates)
+constexpr int kVecBytes = 4 * 512 + 128;               // q k v | gate (channel gates) | scalar gate, beta
 constexpr int kOffBars = 0;                            // uint64 [8]
 constexpr int kOffRed = 64;                            // float [2][8][128]: retrieval, readout
 constexpr int kOffColD = kOffRed + 2 * 8 * 128 * 4;    // float [128] delta_j
@@ -35,6 +35,7 @@ struct DecodeArgs {
     const float *q, *k, *v, *beta, *gate;
     float *y;
     unsigned int *err;
+    StallKnob stall;
 };
 
 __device__ __forceinline__ void row_dup(const float4 *v, int i, uint64_t &xx, uint64_t &zz) {
@@ -63,24 +64,33 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeArgs a) {
     const auto page_of = [&](int h, int slot) {
         return a.pool + (uint64_t)slot * a.slot_bytes + a.layer_off + (uint64_t)h * kPage;
     };
-    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err};
+    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err, a.stall.wait_cycles,
+                        a.stall.withhold_item};
     pipe::run(
         p, bars,
-        [&](int h, int b, int slot, int s) {
+        [&](int h, int b, int slot, int s, int lane) {
             uint8_t *st = stages + (size_t)s * kStage;
             float *vec = (float *)(st + kPage);
             const int hk = h / grp;
-            mbar_arrive_tx(&bars[s], kPage + (a.gate_per_row ? 2048 : 1536));
-            bulk_load(st, page_of(h, slot), kPage, &bars[s]);
-            bulk_load(vec, a.q + ((size_t)b * a.Hk + hk) * 128, 512, &bars[s]);
-            bulk_load(vec + 128, a.k + ((size_t)b * a.Hk + hk) * 128, 512, &bars[s]);
-            bulk_load(vec + 256, a.v + ((size_t)b * a.Hv + h) * 128, 512, &bars[s]);
-            if (a.gate_per_row) bulk_load(vec + 384, a.gate + ((size_t)b * a.Hv + h) * 128, 512, &bars[s]);
+            const size_t u = (size_t)b * a.Hv + h;
+            warp_copy512(vec, a.q + ((size_t)b * a.Hk + hk) * 128, lane);
+            warp_copy512(vec + 128, a.k + ((size_t)b * a.Hk + hk) * 128, lane);
+            warp_copy512(vec + 256, a.v + u * 128, lane);
+            if (a.gate_per_row) warp_copy512(vec + 384, a.gate + u * 128, lane);
+            else if (lane == 1) cp_async4(vec + 512, a.gate + u);
+            if (lane == 0) cp_async4(vec + 513, a.beta + u);
+            cp_async_mbar_arrive(&bars[s]);
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive_tx(&bars[s], kPage);
+                bulk_load(st, page_of(h, slot), kPage, &bars[s]);
+            }
         },
         [&](int h, int b, int slot, int s, bool ok, const auto &refill) {
             const size_t u = (size_t)b * a.Hv + h;
-            const float beta = a.beta[u], gs = a.gate_per_row ? 0.f : a.gate[u];
             float *S = (float *)(stages + (size_t)s * kStage);
+            const float *sv = S + kN;
+            const float beta = sv[513], gs = a.gate_per_row ? 0.f : sv[512];       // staged
             const float *q = S + kN, *k = q + 128, *v = q + 256, *gv = q + 384;
             if (l < 16) {
                 const int i = 16 * w + l;
@@ -175,6 +185,7 @@ stepq_status launch_fp32_decode(const stepq_config *cfg, int layer, float *pool,
     a.gate_per_row = cfg->gate_kind == STEPQ_GATE_CHANNEL;
     a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
     a.err = device_error_word();
+    a.stall = stall_knob();
     int dev = 0, sms = 1, max_smem = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);

@@ -18,6 +18,8 @@
 // page in place in shared memory, and a bulk store writes it back. Every wait
 // is bounded: a stalled copy raises STEPQ_ERR_TIMEOUT and the CTA drains its
 // own copies before returning.
+#include <atomic>
+
 #include "async.cuh"
 #include "device.cuh"
 #include "internal.h"
@@ -491,6 +493,7 @@ struct DecodeArgs {
     float *y;
     float *delta;              // readout: delta_j out; writeback: delta_j in
     unsigned int *err;
+    StallKnob stall;
     int n_stages;
     uint32_t page_region, stage_bytes;
     int fit_iters;
@@ -500,25 +503,29 @@ struct DecodeArgs {
 // into stage s. The writeback loads delta into the v slot and needs no q; the
 // readout needs no w2, wis.
 template <int MODE>
-__device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s) {
+__device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s,
+                                      int lane) {
     uint64_t *bar = &S.bars[s];
     Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
-    const uint32_t nb = S.hbytes[h];
     const int hk = S.hkey[h];
-    constexpr uint32_t vec = MODE == kFused ? 5 * 512 : 4 * 512 - (MODE == kReadout ? 512 : 0);
-    const size_t u = (size_t)b * a.Hv + h;
-    cp_async4(st.gb, a.gate + u);
-    cp_async4(st.gb + 1, a.beta + u);
-    cp_async_mbar_arrive(bar);
-    mbar_arrive_tx(bar, nb + vec);
-    bulk_load(st.page, a.pool + (uint64_t)slot * a.stride + S.hoff[h], nb, bar);
-    if (MODE != kWriteback) bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
-    bulk_load(st.k, a.k + ((size_t)b * a.Hk + hk) * 128, 512, bar);
-    if (MODE != kWriteback) bulk_load(st.v, a.v + ((size_t)b * a.Hv + h) * 128, 512, bar);
-    else bulk_load(st.v, a.delta + ((size_t)b * a.Hv + h) * 128, 512, bar);
+    if (MODE != kWriteback) warp_copy512(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, lane);
+    warp_copy512(st.k, a.k + ((size_t)b * a.Hk + hk) * 128, lane);
+    warp_copy512(st.v, (MODE != kWriteback ? a.v : a.delta) + ((size_t)b * a.Hv + h) * 128, lane);
     if (MODE != kReadout) {
-        bulk_load(st.w2, a.tab.w2 + (size_t)h * 128, 512, bar);
-        bulk_load(st.wis, a.tab.wis + (size_t)h * 128, 512, bar);
+        warp_copy512(st.w2, a.tab.w2 + (size_t)h * 128, lane);
+        warp_copy512(st.wis, a.tab.wis + (size_t)h * 128, lane);
+    }
+    if (lane == 0) {
+        const size_t u = (size_t)b * a.Hv + h;
+        cp_async4(st.gb, a.gate + u);
+        cp_async4(st.gb + 1, a.beta + u);
+    }
+    cp_async_mbar_arrive(bar);
+    __syncwarp();
+    if (lane == 0) {
+        const uint32_t nb = S.hbytes[h];
+        mbar_arrive_tx(bar, nb);
+        bulk_load(st.page, a.pool + (uint64_t)slot * a.stride + S.hoff[h], nb, bar);
     }
 }
 
@@ -674,10 +681,11 @@ __global__ void __launch_bounds__(kThreads, 2) decode_heads_kernel(DecodeArgs a)
         mbar_init_fence();
     }
     __syncthreads();
-    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err};
+    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err, a.stall.wait_cycles,
+                        a.stall.withhold_item};
     pipe::run(
         p, S.bars,
-        [&](int h, int b, int slot, int s) { issue<MODE>(a, S, h, b, slot, s); },
+        [&](int h, int b, int slot, int s, int lane) { issue<MODE>(a, S, h, b, slot, s, lane); },
         [&](int h, int b, int, int s, bool ok, const auto &refill) {
             const size_t u = (size_t)b * a.Hv + h;
             const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
@@ -822,12 +830,16 @@ static stepq_status set_attr(const void *fn, int bytes) {
 }
 
 static int sm_count() {
-    static int n[64];
+    static std::atomic<int> n[64];        // per device; racing first calls store the same value
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev < 0 || dev >= 64) return 1;
-    if (!n[dev]) cudaDeviceGetAttribute(&n[dev], cudaDevAttrMultiProcessorCount, dev);
-    return n[dev] > 0 ? n[dev] : 1;
+    int v = n[dev].load(std::memory_order_relaxed);
+    if (!v) {
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+        n[dev].store(v, std::memory_order_relaxed);
+    }
+    return v > 0 ? v : 1;
 }
 
 stepq_status launch_decode_heads(const stepq_plan *p, int layer, uint8_t *pool, int pool_slots,
@@ -860,6 +872,7 @@ stepq_status launch_decode_heads_mode(const stepq_plan *p, int layer, uint8_t *p
     a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
     a.delta = delta;
     a.err = device_error_word();
+    a.stall = stall_knob();
     a.page_region = (maxb + 127) / 128 * 128;
     a.stage_bytes = a.page_region + hk::kVecBytes;
     // as many stages (2..4) as keep two CTAs per SM

@@ -52,19 +52,21 @@ struct DecodeArgs {
     const float *q, *k, *v, *beta, *gate;
     float *y;
     unsigned int *err;
+    StallKnob stall;
     int n_stages;
     uint32_t page_region, stage_bytes, vec_bytes;
 };
 
 struct Stage {
     uint8_t *page;
-    float *q, *k, *v, *gate;
+    float *q, *k, *v, *gate, *gb;
     __device__ __forceinline__ Stage(uint8_t *base, uint32_t page_region) {
         page = base;
         q = (float *)(base + page_region);
         k = q + 128;
         v = q + 256;
         gate = q + 384;
+        gb = q + 512;       // scalar gate, beta
     }
 };
 
@@ -290,24 +292,32 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(DecodeArgs a, int b
     const auto page_of = [&](int h, int slot) {
         return a.pool + (uint64_t)slot * a.slot_bytes + a.layer_off + (uint64_t)h * a.head_bytes;
     };
-    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err};
+    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err, a.stall.wait_cycles,
+                        a.stall.withhold_item};
     pipe::run(
         p, S.bars,
-        [&](int h, int b, int slot, int s) {
+        [&](int h, int b, int slot, int s, int lane) {
             uint64_t *bar = &S.bars[s];
             const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
             const int hk = h / grp;
-            mbar_arrive_tx(bar, (uint32_t)a.head_bytes + a.vec_bytes);
-            bulk_load(st.page, page_of(h, slot), (uint32_t)a.head_bytes, bar);
-            bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
-            bulk_load(st.k, a.k + ((size_t)b * a.Hk + hk) * 128, 512, bar);
-            bulk_load(st.v, a.v + ((size_t)b * a.Hv + h) * 128, 512, bar);
-            if (a.gate_per_row) bulk_load(st.gate, a.gate + ((size_t)b * a.Hv + h) * 128, 512, bar);
+            const size_t u = (size_t)b * a.Hv + h;
+            warp_copy512(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, lane);
+            warp_copy512(st.k, a.k + ((size_t)b * a.Hk + hk) * 128, lane);
+            warp_copy512(st.v, a.v + u * 128, lane);
+            if (a.gate_per_row) warp_copy512(st.gate, a.gate + u * 128, lane);
+            else if (lane == 1) cp_async4(st.gb, a.gate + u);
+            if (lane == 0) cp_async4(st.gb + 1, a.beta + u);
+            cp_async_mbar_arrive(bar);
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive_tx(bar, (uint32_t)a.head_bytes);
+                bulk_load(st.page, page_of(h, slot), (uint32_t)a.head_bytes, bar);
+            }
         },
         [&](int h, int b, int, int s, bool ok, const auto &refill) {
             const size_t u = (size_t)b * a.Hv + h;
-            const float beta = a.beta[u], gs = a.gate_per_row ? 0.f : a.gate[u];
             const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
+            const float beta = st.gb[1], gs = a.gate_per_row ? 0.f : st.gb[0];    // staged
             float *y_out = a.y + u * 128;
             if (bits == 8) return decode_item<8>(t, S, st, gs, a.gate_per_row, beta, y_out, ok, refill);
             if (bits == 6) return decode_item<6>(t, S, st, gs, a.gate_per_row, beta, y_out, ok, refill);
@@ -341,9 +351,10 @@ stepq_status launch_intb_decode(const stepq_config *cfg, int bits, int layer, ui
     a.gate_per_row = cfg->gate_kind == STEPQ_GATE_CHANNEL;
     a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
     a.err = device_error_word();
+    a.stall = stall_knob();
     a.page_region = (uint32_t)((hb + 127) / 128 * 128);
     a.vec_bytes = a.gate_per_row ? 2048 : 1536;
-    a.stage_bytes = a.page_region + 2048;
+    a.stage_bytes = a.page_region + 2048 + 128;
     int stages = (int)((113 * 1024 - ib::kOffStages) / a.stage_bytes);
     stages = stages < 2 ? 2 : (stages > 4 ? 4 : stages);
     a.n_stages = stages;

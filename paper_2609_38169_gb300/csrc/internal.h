@@ -159,6 +159,14 @@ stepq_status launch_validate_slots_static(const int32_t *slots, int B, int pool_
                                           int32_t *status, cudaStream_t s);
 stepq_status read_device_error(cudaStream_t s);
 unsigned int *device_error_word();   // address of the current device's sticky error word
+// Test switch of the pipelined decode kernels (stepq_debug_stall): the bound of
+// every wait in SM cycles and an item whose copies never start (-1: none).
+struct StallKnob {
+    long long wait_cycles;
+    int withhold_item;
+};
+StallKnob stall_knob();
+stepq_status set_stall_knob(long long wait_cycles, int withhold_item);
 
 size_t intb_head_bytes(int bits);
 

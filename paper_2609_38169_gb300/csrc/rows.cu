@@ -25,7 +25,7 @@
 namespace stepq {
 namespace rk {
 
-constexpr int kVecBytes = 7 * 512;                     // q k v gate w2 wis | row slots
+constexpr int kVecBytes = 7 * 512 + 128;               // q k v gate w2 wis | row slots | beta
 
 // ------------------------------------------------------------ shared layout
 constexpr int kOffBars = 0;                            // uint64 [8]
@@ -78,6 +78,7 @@ struct Stage {
     uint8_t *page;
     float *q, *k, *v, *gate, *w2, *wis;
     uint32_t *slot;     // s-th stored row of the head: offset | width << 16 | row << 24
+    float *beta;
     __device__ __forceinline__ Stage(uint8_t *base, uint32_t page_region) {
         page = base;
         q = (float *)(base + page_region);
@@ -87,6 +88,7 @@ struct Stage {
         w2 = q + 512;
         wis = q + 640;
         slot = (uint32_t *)(q + 768);
+        beta = q + 896;
     }
 };
 
@@ -185,6 +187,7 @@ struct DecodeArgs {
     float *y;
     float *delta;              // readout: delta_j out; writeback: delta_j in
     unsigned int *err;
+    StallKnob stall;
     int n_stages;
     uint32_t page_region, stage_bytes;
     int fit_iters;
@@ -195,24 +198,29 @@ struct DecodeArgs {
 enum : int { kFused = 0, kReadout = 1, kWriteback = 2 };
 
 template <int MODE>
-__device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s) {
+__device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s,
+                                      int lane) {
     uint64_t *bar = &S.bars[s];
     Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
-    const uint32_t nb = S.hbytes[h];
     const int hk = S.hkey[h];
-    constexpr uint32_t vec = MODE == kFused ? kVecBytes : kVecBytes - (MODE == kReadout ? 1024 : 512);
-    mbar_arrive_tx(bar, nb + vec);
-    bulk_load(st.page, a.pool + (uint64_t)slot * a.stride + S.hoff[h], nb, bar);
-    if (MODE != kWriteback) bulk_load(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, 512, bar);
-    bulk_load(st.k, a.k + ((size_t)b * a.Hk + hk) * 128, 512, bar);
-    if (MODE != kWriteback) bulk_load(st.v, a.v + ((size_t)b * a.Hv + h) * 128, 512, bar);
-    else bulk_load(st.v, a.delta + ((size_t)b * a.Hv + h) * 128, 512, bar);
-    bulk_load(st.gate, a.gate + ((size_t)b * a.Hv + h) * 128, 512, bar);
+    const size_t u = (size_t)b * a.Hv + h;
+    if (MODE != kWriteback) warp_copy512(st.q, a.q + ((size_t)b * a.Hk + hk) * 128, lane);
+    warp_copy512(st.k, a.k + ((size_t)b * a.Hk + hk) * 128, lane);
+    warp_copy512(st.v, (MODE != kWriteback ? a.v : a.delta) + u * 128, lane);
+    warp_copy512(st.gate, a.gate + u * 128, lane);
     if (MODE != kReadout) {
-        bulk_load(st.w2, a.tab.w2 + (size_t)h * 128, 512, bar);
-        bulk_load(st.wis, a.tab.wis + (size_t)h * 128, 512, bar);
+        warp_copy512(st.w2, a.tab.w2 + (size_t)h * 128, lane);
+        warp_copy512(st.wis, a.tab.wis + (size_t)h * 128, lane);
     }
-    bulk_load(st.slot, a.tab.row_slot + (size_t)h * 128, 512, bar);
+    warp_copy512(st.slot, a.tab.row_slot + (size_t)h * 128, lane);
+    if (lane == 0) cp_async4(st.beta, a.beta + u);
+    cp_async_mbar_arrive(bar);
+    __syncwarp();
+    if (lane == 0) {
+        const uint32_t nb = S.hbytes[h];
+        mbar_arrive_tx(bar, nb);
+        bulk_load(st.page, a.pool + (uint64_t)slot * a.stride + S.hoff[h], nb, bar);
+    }
 }
 
 // Z of row pair m (columns 4l..4l+3): c_j q_ij (exact) for integer rows, the
@@ -611,13 +619,14 @@ __global__ void __launch_bounds__(kThreads, 2) decode_rows_kernel(DecodeArgs a) 
         mbar_init_fence();
     }
     __syncthreads();
-    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err};
+    const pipe::Shape p{a.items, a.nb, a.n_stages, a.slots, a.pool_slots, a.err, a.stall.wait_cycles,
+                        a.stall.withhold_item};
     pipe::run(
-        p, S.bars, [&](int h, int b, int slot, int s) { issue<MODE>(a, S, h, b, slot, s); },
+        p, S.bars, [&](int h, int b, int slot, int s, int lane) { issue<MODE>(a, S, h, b, slot, s, lane); },
         [&](int h, int b, int, int s, bool ok, const auto &refill) {
             const size_t u = (size_t)b * a.Hv + h;
-            const float beta = a.beta[u];
             const Stage st(S.stages + (size_t)s * a.stage_bytes, a.page_region);
+            const float beta = *st.beta;                   // staged with the page
             return decode_item<MODE>(t, S, st, beta, MODE == kWriteback ? nullptr : a.y + u * 128,
                                      MODE == kReadout ? a.delta + u * 128 : nullptr, a.fit_iters, ok,
                                      refill);
@@ -661,6 +670,7 @@ stepq_status launch_decode_rows_mode(const stepq_plan *p, int layer, uint8_t *po
     a.q = q; a.k = k; a.v = v; a.beta = beta; a.gate = gate; a.y = y;
     a.delta = delta;
     a.err = device_error_word();
+    a.stall = stall_knob();
     a.page_region = (maxb + 127) / 128 * 128;
     a.stage_bytes = a.page_region + rk::kVecBytes;
     // as many stages (2..4) as keep two CTAs per SM

@@ -13,6 +13,7 @@
 // c is fitted from the clip-free start
 // max_i fp32(fp32(|X_ij| rho_i) / qmax_i) by `fit_iters` fixed-code
 // least-squares updates.
+#include <atomic>
 #include <cstdio>
 
 #include "device.cuh"
@@ -390,7 +391,7 @@ __global__ void __launch_bounds__(kThreads, 2) distortion_kernel(DistArgs a) {
 }
 
 // ------------------------------------------------------------------ launchers
-static bool g_attr_set[64];
+static std::atomic<bool> g_attr_set[64];   // per device; setting the attributes twice is harmless
 
 static stepq_status prepare(int dev) {
     if (dev < 0) cudaGetDevice(&dev);

@@ -121,3 +121,38 @@ def test_too_many_heads_is_refused(torch):
         A.stepq_decode_step(plan, 0, pool_d, slots, z, z, zv, beta, gate, zv.clone())
     assert torch.equal(pool_d, before)
     assert A.stepq_device_error() == 0
+
+
+@pytest.mark.parametrize("name,withhold", [("gqa", 0), ("gqa", 37), ("channel", 5)])
+def test_bounded_wait_runs_out_and_recovers(torch, name, withhold):
+    """Failure detection without a fault: a test switch makes the producer skip
+    the copies of one item, so that item's stage barrier never completes. With
+    the wait bound lowered to 1e5 cycles the kernel gives up, every CTA returns,
+    and the launch reports STEPQ_ERR_TIMEOUT through the sticky error word. The
+    next, normal step on the same context matches the oracle."""
+    wl = W.WORKLOADS[name].replace(pool_slots=8)
+    B = 4
+    S = W.random_states(wl, B * wl.hv, seed=3).reshape(B, wl.hv, 128, 128)
+    cfg, plan, oplan, _ = plans(wl)
+    slots = np.array([6, 1, 4, 2], np.int32)
+    pool_o = np.zeros(wl.pool_slots * oplan.slot_stride, np.uint8)
+    O.pool_encode(oplan, pool_o, 0, slots, S)
+    pool_d = torch.from_numpy(pool_o.copy()).cuda()
+    inp = W.step_inputs(wl, W.model_params(wl), W.STREAM_DECODE, 0, 0, batch=B)
+    q, k, v, beta, gate, slots_d = to_dev(inp.q, inp.k, inp.v, inp.beta, inp.gate, slots)
+    y_d = torch.empty((B, wl.hv, 128), dtype=torch.float32, device="cuda")
+    A.stepq_debug_stall(100_000, withhold)
+    try:
+        A.stepq_decode_step(plan, 0, pool_d, slots_d, q, k, v, beta, gate, y_d)
+        assert A.stepq_device_error() == 8                                      # STEPQ_ERR_TIMEOUT
+    finally:
+        A.stepq_debug_stall()
+    pool_d.copy_(torch.from_numpy(pool_o))
+    A.stepq_decode_step(plan, 0, pool_d, slots_d, q, k, v, beta, gate, y_d)
+    y_o = O.pool_step(oplan, pool_o, 0, slots, inp)
+    t = Tally()
+    compare_y(t, y_d.cpu().numpy(), y_o)
+    compare_pools(t, pool_d.cpu().numpy(), pool_o, oplan, 0, slots)
+    print(name, t.summary())
+    t.check()
+    assert A.stepq_device_error() == 0

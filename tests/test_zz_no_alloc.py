@@ -31,8 +31,9 @@ def test_noalloc_slot_check_matches_scratch_version():
         list(range(0, 5000, 3)),         # many distinct
         [4999, 4999],                    # a repeat at the top bit of the last word
     ]
+    expected = [0, 3, 2, 0, 3]           # STEPQ_OK, _DUP_SLOT, _SLOT_RANGE, _OK, _DUP_SLOT
     for _round in range(2):              # two calls in a row per case, then all again
-        for case in cases:
+        for case, want in zip(cases, expected):
             slots = torch.tensor(case, dtype=torch.int32, device=dev)
             ref = torch.full((1,), -1, dtype=torch.int32, device=dev)
             got = torch.full((1,), -1, dtype=torch.int32, device=dev)
@@ -45,7 +46,7 @@ def test_noalloc_slot_check_matches_scratch_version():
                                                       pool_slots, C.c_void_p(got.data_ptr()),
                                                       stream) == 0
                 torch.cuda.synchronize(dev)
-                assert int(got.item()) == int(ref.item()), (case, int(got.item()), int(ref.item()))
+                assert int(got.item()) == int(ref.item()) == want, (case, int(got.item()), int(ref.item()))
     # a pool beyond the fixed array is refused before any work
     one = torch.zeros(1, dtype=torch.int32, device=dev)
     assert L.stepq_validate_slots_noalloc(C.c_void_p(one.data_ptr()), 1, (1 << 20) + 1,
