@@ -133,9 +133,9 @@ void stepq_plan_destroy(stepq_plan *plan);
 /* ----------------------------------------------------------------- device path
  * Pool: device, pool_slots * slot_stride bytes, 256-byte aligned. Slot page s
  * starts at pool + s * slot_stride and holds every (layer, head) segment:
- *   integer head unit: r[128] fp16 | c[128] fp16 | codes in band-major chunks:
- *                      for band w = 0..7 (rows 16w..16w+15) and column j, the
- *                      band's 16 codes of column j in 2b bytes
+ *   integer head unit: r[128] fp16 | c[128] fp16 | codes in chunks: the 16
+ *                      codes of band g (rows 16g..16g+15) in column j take 2b
+ *                      bytes, chunk index ((j / 4) * 8 + g) * 4 + j % 4
  *   FP16 pivot head:   the same chunk order of fp16 values (32 bytes per chunk)
  *   row-unit head:     r[128] fp16 | c[128] fp16 | the rows, 16*b_i bytes each
  *                      (b_i = 16: fp16 row), stored by decreasing width, rows of

@@ -26,11 +26,12 @@
  *  - codes are stored offset-binary u = q + 2^(b-1), LSB-first per row.
  *
  * Page layout of one head (all pieces 16-byte multiples):
- *   integer head unit: r[128] fp16 | c[128] fp16 | codes in band-major order:
- *                      for band w = 0..7 (rows 16w..16w+15), for column j,
- *                      the 16 codes of rows 16w.. in that column (2b bytes)
- *   pivot head unit:   the same band-major order of fp16 values (32 bytes
- *                      per band column), no scales
+ *   integer head unit: r[128] fp16 | c[128] fp16 | codes in chunks of the 16
+ *                      codes of one band of rows (16g..16g+15) in one column
+ *                      (2b bytes), ordered by column group (columns 4t..4t+3),
+ *                      then band g, then column within the group
+ *   pivot head unit:   the same chunk order of fp16 values (32 bytes per
+ *                      chunk), no scales
  *   row-unit head:     r[128] fp16 | c[128] fp16 | then the rows, each 16 b_i
  *                      bytes with the codes of columns 0..127 (b_i = 16 marks
  *                      an FP16 pivot row, 256 bytes), stored by decreasing
@@ -100,7 +101,7 @@ static size_t elem_stream(int unit_kind, const int8_t *rb, int i, int j, int *bi
     int b = rb[i];
     if (unit_kind == OR_UNIT_HEAD) {
         size_t base = is_pivot_head(unit_kind, rb) ? 0 : 512;
-        size_t chunk = (size_t)(i / 16) * OR_D + (size_t)j;        /* band-major chunks */
+        size_t chunk = ((size_t)(j / 4) * 8 + (size_t)(i / 16)) * 4 + (size_t)(j % 4);
         *bitpos = (i % 16) * b;
         return base + chunk * 2 * (size_t)b;
     }

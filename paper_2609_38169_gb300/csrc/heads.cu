@@ -1,23 +1,28 @@
 // Head-unit (GDN) kernels: the persistent, bulk-async pipelined decode step and
-// the pack/unpack kernels for head pages stored in band-major order.
+// the pack/unpack kernels of head pages.
 //
-// Tile mapping: warp w owns the band of key rows 16w..16w+15; lane l owns the
-// value columns l, l+32, l+64, l+96. A thread holds a 16 x 4 register tile as
-// eight row pairs (rows 2m, 2m+1 of its band) per column, each pair one packed
-// f32x2 register: per-row constants of a row pair are adjacent in shared
-// memory (one 128-bit broadcast load serves two pairs), and the two codes of a
-// pair are adjacent in the band-major chunk. Every column reduction needs one
-// cross-warp step and the single row reduction (m_i) stays inside a warp. In
-// the page a thread's 16 codes of one column are one 2b-byte chunk and
-// consecutive lanes read consecutive chunks (no shared-memory bank conflicts).
+// Tile mapping: warp w owns the value columns 16w..16w+15 of the head, all 128
+// key rows. Lane l = 8 cg + rg holds the 16 rows 16rg..16rg+15 (band rg) of the
+// 4 columns 16w + 4cg .. 16w + 4cg + 3, as eight row pairs (rows 2m, 2m+1 of
+// its band) per column, each pair one packed f32x2 register. So every column
+// reduction (retrieval, readout, column maximum, least squares) stays inside a
+// warp: a three-level shuffle reduce-scatter over the 8 lanes of a column
+// group, whose result lane rg holds for column rg >> 1 of its group. Only the
+// row reduction of the row factors crosses warps, through shared memory.
+//
+// Page chunks: the 16 codes of band g in column j take 2b bytes; chunk index
+// ((j / 4) * 8 + g) * 4 + j % 4, so thread tid's four chunks are the 8b
+// contiguous bytes of block tid and the 32 lanes of a warp read 32 consecutive
+// blocks (no shared-memory bank conflicts beyond the minimum wavefronts).
+// Per-row constants sit in shared memory with a pad of 4 floats after every
+// band of 16 rows, so the 8 bands a warp reads hit distinct banks.
 //
 // Decode pipeline (App. C.3 steps 1-7 per head): each persistent CTA walks its
-// (head, slot) items, head-major so that concurrently resident CTAs mostly run
-// the code of one head width; one thread keeps up to S-1 pages in flight with
-// bulk copies completing on per-stage mbarriers, the CTA updates and refits the
-// page in place in shared memory, and a bulk store writes it back. Every wait
-// is bounded: a stalled copy raises STEPQ_ERR_TIMEOUT and the CTA drains its
-// own copies before returning.
+// (head, slot) items, head-major; the last warp keeps up to S-1 pages in flight
+// (pipeline.cuh), the CTA updates and refits the page in place in shared
+// memory, and a bulk store writes it back. CTA barriers per item: one after the
+// row constants (which also agrees on the stage's copies), two around the row
+// factors, one before the store.
 #include <atomic>
 
 #include "async.cuh"
@@ -30,28 +35,23 @@ namespace stepq {
 namespace hk {
 
 constexpr int kVecBytes = 5 * 512 + 128;               // q k v w2 wis | gate, beta per stage
+constexpr int kPad = 160;                              // padded per-row array: 8 bands x (16 + 4)
 
 // ------------------------------------------------------------ shared layout
 constexpr int kOffBars = 0;                            // uint64 [8]
-constexpr int kOffFlags = 64;                          // int [16]
-constexpr int kOffRed = 128;                           // float [3][8][128] cross-warp partials
-constexpr int kOffColC = kOffRed + 3 * 8 * 128 * 4;    // float [128] c_j (start / iterate)
-constexpr int kOffColX = kOffColC + 512;               // float [128] max_i |X'_ij|
-constexpr int kOffColM = kOffColX + 512;               // u32 [128] bits of max_i |X'_ij| (atomic)
-constexpr int kOffColD = kOffColM + 512;               // float2 [128] (delta_j, delta_j)
-constexpr int kOffColG = kOffColD + 1024;              // float2 [128] (1/c_j, 1/c_j)
-constexpr int kOffRows = kOffColG + 1024;              // float [6][128] per-row constants
+constexpr int kOffRed = 128;                           // float [8][128] row partial sums per warp
+constexpr int kOffRows = kOffRed + 8 * 128 * 4;        // float [6][kPad] per-row constants
 constexpr int kMaxHv = 256;                            // value heads per layer (launch check)
-constexpr int kOffHead = kOffRows + 6 * 512;           // u64 off | u32 bytes | u8 bits | u8 key head
+constexpr int kOffHead = kOffRows + 6 * kPad * 4;      // u64 off | u32 bytes | u8 bits | u8 key head
 constexpr int kOffStages = (kOffHead + kMaxHv * 14 + 127) / 128 * 128;
+
+// padded index of row i in a per-row array
+__host__ __device__ constexpr int prow(int i) { return 20 * (i >> 4) + (i & 15); }
 
 struct Smem {
     uint64_t *bars;
-    int *flags;
-    float *red, *colC, *colX;
-    uint32_t *colM;
-    float2 *colD, *colG;
-    // per-row constants: kappa_i = k_i a_i, beta k_i / a_i, q_i a_i, a_i,
+    float *red;
+    // per-row constants (padded): kappa_i = k_i a_i, beta k_i / a_i, q_i a_i, a_i,
     // rho_i a_i and the least-squares weight alpha_i = w_i^2 r_i^2
     float *rKap, *rBkp, *rQa, *rA, *rRho, *rAl;
     uint64_t *hoff;
@@ -60,19 +60,13 @@ struct Smem {
     uint8_t *stages;
     __device__ __forceinline__ explicit Smem(uint8_t *s) {
         bars = (uint64_t *)(s + kOffBars);
-        flags = (int *)(s + kOffFlags);
         red = (float *)(s + kOffRed);
-        colC = (float *)(s + kOffColC);
-        colX = (float *)(s + kOffColX);
-        colM = (uint32_t *)(s + kOffColM);
-        colD = (float2 *)(s + kOffColD);
-        colG = (float2 *)(s + kOffColG);
         rKap = (float *)(s + kOffRows);
-        rBkp = rKap + 128;
-        rQa = rKap + 256;
-        rA = rKap + 384;
-        rRho = rKap + 512;
-        rAl = rKap + 640;
+        rBkp = rKap + kPad;
+        rQa = rKap + 2 * kPad;
+        rA = rKap + 3 * kPad;
+        rRho = rKap + 4 * kPad;
+        rAl = rKap + 5 * kPad;
         hoff = (uint64_t *)(s + kOffHead);
         hbytes = (uint32_t *)(s + kOffHead + kMaxHv * 8);
         hbits = s + kOffHead + kMaxHv * 12;
@@ -96,87 +90,112 @@ struct Stage {
 };
 
 struct T {   // thread coordinates
-    int tid, w, l;
+    int tid, w, l, rg, cg;
     __device__ __forceinline__ T() {
         tid = threadIdx.x;
         w = tid >> 5;
         l = tid & 31;
+        rg = l & 7;
+        cg = l >> 3;
     }
-    __device__ __forceinline__ int row(int r) const { return 16 * w + r; }
-    __device__ __forceinline__ int col(int c) const { return l + 32 * c; }
+    __device__ __forceinline__ int row(int r) const { return 16 * rg + r; }
+    __device__ __forceinline__ int col(int c) const { return 16 * w + 4 * cg + c; }
+    // the column whose reduced value this lane holds after a reduce-scatter
+    __device__ __forceinline__ int own_col() const { return col(rg >> 1); }
 };
 
-// Row-pair constants m = 2p, 2p+1 of the warp's band from one 128-bit load.
+// Row-pair constants m = 2p, 2p+1 of the thread's band from one 128-bit load.
 __device__ __forceinline__ void row_pairs(const float *v, const T &t, int p, uint64_t &lo, uint64_t &hi) {
-    const uint4 q = *(const uint4 *)&v[t.row(4 * p)];
+    const uint4 q = *(const uint4 *)&v[20 * t.rg + 4 * p];
     lo = u2pair(q.x, q.y);
     hi = u2pair(q.z, q.w);
 }
-__device__ __forceinline__ uint64_t col_pair(const float2 *v, int j) {
-    return *(const uint64_t *)&v[j];
+
+// ---- warp reductions over the 8 lanes of a column group (lane bits 0-2) ----
+// Lane rg returns the total over the group of v[rg >> 1].
+__device__ __forceinline__ float col_sum_scatter(const float (&v)[4], int rg) {
+    const bool b2 = rg & 4, b1 = rg & 2;
+    const float a0 = (b2 ? v[2] : v[0]) + __shfl_xor_sync(0xffffffffu, b2 ? v[0] : v[2], 4);
+    const float a1 = (b2 ? v[3] : v[1]) + __shfl_xor_sync(0xffffffffu, b2 ? v[1] : v[3], 4);
+    const float a = (b1 ? a1 : a0) + __shfl_xor_sync(0xffffffffu, b1 ? a0 : a1, 2);
+    return a + __shfl_xor_sync(0xffffffffu, a, 1);
+}
+__device__ __forceinline__ float col_max_scatter(const float (&v)[4], int rg) {
+    const bool b2 = rg & 4, b1 = rg & 2;
+    const float a0 = fmaxf(b2 ? v[2] : v[0], __shfl_xor_sync(0xffffffffu, b2 ? v[0] : v[2], 4));
+    const float a1 = fmaxf(b2 ? v[3] : v[1], __shfl_xor_sync(0xffffffffu, b2 ? v[1] : v[3], 4));
+    const float a = fmaxf(b1 ? a1 : a0, __shfl_xor_sync(0xffffffffu, b1 ? a0 : a1, 2));
+    return fmaxf(a, __shfl_xor_sync(0xffffffffu, a, 1));
+}
+// Two values per column (least-squares numerator and denominator).
+__device__ __forceinline__ void col_sum2_scatter(const float (&n)[4], const float (&d)[4], int rg,
+                                                 float &no, float &dout) {
+    const bool b2 = rg & 4, b1 = rg & 2;
+    const float n0 = (b2 ? n[2] : n[0]) + __shfl_xor_sync(0xffffffffu, b2 ? n[0] : n[2], 4);
+    const float n1 = (b2 ? n[3] : n[1]) + __shfl_xor_sync(0xffffffffu, b2 ? n[1] : n[3], 4);
+    const float d0 = (b2 ? d[2] : d[0]) + __shfl_xor_sync(0xffffffffu, b2 ? d[0] : d[2], 4);
+    const float d1 = (b2 ? d[3] : d[1]) + __shfl_xor_sync(0xffffffffu, b2 ? d[1] : d[3], 4);
+    const float na = (b1 ? n1 : n0) + __shfl_xor_sync(0xffffffffu, b1 ? n0 : n1, 2);
+    const float da = (b1 ? d1 : d0) + __shfl_xor_sync(0xffffffffu, b1 ? d0 : d1, 2);
+    no = na + __shfl_xor_sync(0xffffffffu, na, 1);
+    dout = da + __shfl_xor_sync(0xffffffffu, da, 1);
+}
+// The value of column c of the thread's group from the lane that holds it.
+__device__ __forceinline__ float col_gather(float v, const T &t, int c) {
+    return __shfl_sync(0xffffffffu, v, (t.l & 24) | (2 * c));
 }
 
-// Byte offset of the band-major chunk (band w, column j) in a head page.
-template <int B>
-__device__ __forceinline__ int chunk_off(int w, int j) {
-    return (B == kPivot ? 0 : 512) + (w * 128 + j) * 2 * B;
+// ---- row reduction over the 4 lanes of a band (lane bits 3-4) ----
+// 16 per-row partials in, 4 out: rows 8 (cg & 1) + 4 (cg >> 1) + t of the band.
+__device__ __forceinline__ void row_sum_scatter(const float (&v)[16], int cg, float (&out)[4]) {
+    float a8[8];
+    const bool b0 = cg & 1, b1 = cg & 2;
+#pragma unroll
+    for (int t = 0; t < 8; t++)
+        a8[t] = (b0 ? v[8 + t] : v[t]) + __shfl_xor_sync(0xffffffffu, b0 ? v[t] : v[8 + t], 8);
+#pragma unroll
+    for (int t = 0; t < 4; t++)
+        out[t] = (b1 ? a8[4 + t] : a8[t]) + __shfl_xor_sync(0xffffffffu, b1 ? a8[t] : a8[4 + t], 16);
 }
 
-// ---- chunk (un)packing: 16 codes (rows of one band) of one column ----
+// ---- page blocks: thread tid's four chunks, 8B contiguous bytes ----
 template <int B>
-__device__ __forceinline__ void load_chunk(const uint8_t *p, uint32_t (&wd)[8]) {
-    if (B == 2) {
-        wd[0] = *(const uint32_t *)p;
-    } else if (B == 4) {
-        uint2 a = *(const uint2 *)p;
-        wd[0] = a.x; wd[1] = a.y;
-    } else if (B == 6) {
-        const uint32_t *q = (const uint32_t *)p;
-        wd[0] = q[0]; wd[1] = q[1]; wd[2] = q[2];
-    } else if (B == 8) {
-        uint4 a = *(const uint4 *)p;
-        wd[0] = a.x; wd[1] = a.y; wd[2] = a.z; wd[3] = a.w;
-    } else {
-        uint4 a = ((const uint4 *)p)[0], b = ((const uint4 *)p)[1];
-        wd[0] = a.x; wd[1] = a.y; wd[2] = a.z; wd[3] = a.w;
-        wd[4] = b.x; wd[5] = b.y; wd[6] = b.z; wd[7] = b.w;
+__device__ __forceinline__ uint8_t *block_ptr(uint8_t *page, int tid) {
+    return page + (B == kPivot ? 0 : 512) + tid * 8 * B;
+}
+template <int B>
+__device__ __forceinline__ void load_block(const uint8_t *p, uint32_t (&wd)[2 * B]) {
+#pragma unroll
+    for (int k = 0; k < B / 2; k++) {
+        const uint4 a = ((const uint4 *)p)[k];
+        wd[4 * k] = a.x; wd[4 * k + 1] = a.y; wd[4 * k + 2] = a.z; wd[4 * k + 3] = a.w;
     }
 }
-
 template <int B>
-__device__ __forceinline__ void store_chunk(uint8_t *p, const uint32_t (&wd)[8]) {
-    if (B == 2) {
-        *(uint32_t *)p = wd[0];
-    } else if (B == 4) {
-        *(uint2 *)p = make_uint2(wd[0], wd[1]);
-    } else if (B == 6) {
-        uint32_t *q = (uint32_t *)p;
-        q[0] = wd[0]; q[1] = wd[1]; q[2] = wd[2];
-    } else if (B == 8) {
-        *(uint4 *)p = make_uint4(wd[0], wd[1], wd[2], wd[3]);
-    } else {
-        ((uint4 *)p)[0] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
-        ((uint4 *)p)[1] = make_uint4(wd[4], wd[5], wd[6], wd[7]);
-    }
+__device__ __forceinline__ void store_block(uint8_t *p, const uint32_t (&wd)[2 * B]) {
+#pragma unroll
+    for (int k = 0; k < B / 2; k++)
+        ((uint4 *)p)[k] = make_uint4(wd[4 * k], wd[4 * k + 1], wd[4 * k + 2], wd[4 * k + 3]);
 }
 
 // Scale of the high code of a pair as placed by code_pair (2^B, or 1 for B = 8).
 template <int B>
 __host__ __device__ constexpr float hi_scale() { return B == 8 ? 1.0f : 1.0f / (float)(1 << B); }
 
-// Codes 2m and 2m+1 of a chunk as the bit patterns of the floats
+// Codes 2m and 2m+1 of chunk c of a block as the bit patterns of the floats
 // 1.5*2^23 + u_lo and 1.5*2^23 + u_hi * 2^B (B = 8: both at the bottom): the
 // codes are dropped into the zero low mantissa bits of the constant, one logic
 // op each (after at most one shift per pair).
 template <int B>
-__device__ __forceinline__ uint64_t code_pair(const uint32_t (&wd)[8], int m) {
+__device__ __forceinline__ uint64_t code_pair(const uint32_t (&wd)[2 * B], int c, int m) {
+    constexpr int W = B / 2;                  // words per chunk
     if (B == 8) {
-        const uint32_t w = wd[m >> 1];
+        const uint32_t w = wd[c * W + (m >> 1)];
         const uint32_t sel = 0x7650u + 2u * (uint32_t)(m & 1);
         return u2pair(__byte_perm(w, kMagicBits, sel), __byte_perm(w, kMagicBits, sel + 1u));
     }
     constexpr uint32_t mask = (1u << B) - 1u;
-    const int p = 2 * m * B, k = p >> 5, s = p & 31;
+    const int p = 2 * m * B, k = c * W + (p >> 5), s = p & 31;
     uint32_t win;
     if (s == 0)
         win = wd[k];
@@ -187,7 +206,7 @@ __device__ __forceinline__ uint64_t code_pair(const uint32_t (&wd)[8], int m) {
     return u2pair(and_or(win, mask, kMagicBits), and_or(win, mask << B, kMagicBits));
 }
 
-// Sum over the 16 codes of the chunk of (0x4B400000 << s) and of the parts
+// Sum over the 16 codes of a chunk of (0x4B400000 << s) and of the parts
 // shifted into the next word, i.e. what pack_codes adds besides the codes.
 __host__ __device__ constexpr uint32_t pack_bias(int B, int k) {
     uint32_t b = 0;
@@ -200,24 +219,24 @@ __host__ __device__ constexpr uint32_t pack_bias(int B, int k) {
 }
 
 // 16 offset-binary codes given as the float bit patterns 0x4B400000 | u_r,
-// packed LSB-first into the chunk words. The high bits are the same constant
-// for every code, so each word is the plain sum of the shifted patterns minus
-// the shifted constants (mod 2^32): one shift-add per code.
+// packed LSB-first into the words of chunk c. The high bits are the same
+// constant for every code, so each word is the plain sum of the shifted
+// patterns minus the shifted constants (mod 2^32): one shift-add per code.
 template <int B>
-__device__ __forceinline__ void pack_codes(const uint32_t (&f)[16], uint32_t (&wd)[8]) {
+__device__ __forceinline__ void pack_codes(const uint32_t (&f)[16], uint32_t (&wd)[2 * B], int c) {
+    constexpr int W = B / 2;
     if (B == 8) {
 #pragma unroll
         for (int t = 0; t < 4; t++) {
             const uint32_t lo = __byte_perm(f[4 * t], f[4 * t + 1], 0x0040);
             const uint32_t hi = __byte_perm(f[4 * t + 2], f[4 * t + 3], 0x0040);
-            wd[t] = __byte_perm(lo, hi, 0x5410);
+            wd[c * W + t] = __byte_perm(lo, hi, 0x5410);
         }
         return;
     }
-    constexpr int NW = B / 2;
-    uint32_t acc[NW];
+    uint32_t acc[W];
 #pragma unroll
-    for (int k = 0; k < NW; k++) acc[k] = 0u - pack_bias(B, k);
+    for (int k = 0; k < W; k++) acc[k] = 0u - pack_bias(B, k);
 #pragma unroll
     for (int r = 0; r < 16; r++) {
         const int p = r * B, k = p >> 5, s = p & 31;
@@ -225,17 +244,7 @@ __device__ __forceinline__ void pack_codes(const uint32_t (&f)[16], uint32_t (&w
         if (s + B > 32) acc[k + 1] += f[r] >> (32 - s);
     }
 #pragma unroll
-    for (int k = 0; k < NW; k++) wd[k] = acc[k];
-}
-
-// Cross-warp column reduction of NR values per thread column (4 columns per
-// thread, 8 warps) into partial region `reg0` and the following ones.
-template <int NR>
-__device__ __forceinline__ void cols_to_red(const T &t, float *red, int reg0, const float (&v)[NR][4]) {
-#pragma unroll
-    for (int k = 0; k < NR; k++)
-#pragma unroll
-        for (int c = 0; c < 4; c++) red[((reg0 + k) * 8 + t.w) * 128 + t.col(c)] = v[k][c];
+    for (int k = 0; k < W; k++) wd[c * W + k] = acc[k];
 }
 
 // Per-row sums over the thread's 4 columns of |value|, for the row pair's
@@ -247,7 +256,7 @@ __device__ __forceinline__ void abs_row_sums(const uint64_t (&x)[4], float &lo, 
 
 // Least-squares sums of the thread's columns: n_j += alpha_i z_ij X'_ij and
 // d_j += alpha_i z_ij^2 with z_ij = rne(X'_ij gamma_j) (one rounding of the
-// exact product), clamped to +-qmax when CLIP (App. C.1).
+// product), clamped to +-qmax when CLIP (App. C.1).
 template <int B, bool CLIP>
 __device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_t (&x2)[8][4],
                                         const uint64_t (&g)[4], uint64_t (&n)[4], uint64_t (&d)[4]) {
@@ -263,7 +272,7 @@ __device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_
             const uint64_t al = h ? ahi : alo;
 #pragma unroll
             for (int c = 0; c < 4; c++) {
-                uint64_t q = fadd2(ffma2(x2[m][c], g[c], M2), nM2);   // rne of the exact product
+                uint64_t q = fadd2(ffma2(x2[m][c], g[c], M2), nM2);   // rne of the product
                 if (CLIP) q = clamp2(q, fqm);
                 const uint64_t aq = fmul2(al, q);
                 n[c] = ffma2(aq, x2[m][c], n[c]);
@@ -274,70 +283,75 @@ __device__ __forceinline__ void ls_sums(const T &t, const Smem &S, const uint64_
 }
 
 // Final codes q_ij = rne(X'_ij gamma_j) with the stored scales (clamped when
-// CLIP), packed into the page chunks.
+// CLIP), packed into the thread's page block.
 template <int B, bool CLIP>
-__device__ __forceinline__ void final_codes(const T &t, const Smem &S, uint8_t *page,
-                                            const uint64_t (&x2)[8][4]) {
+__device__ __forceinline__ void final_codes(const T &t, uint8_t *page, const uint64_t (&x2)[8][4],
+                                            const uint64_t (&g)[4]) {
     constexpr float fqm = (float)((1 << (B - 1)) - 1);
     constexpr float fmb = kMagic + (float)(1 << (B - 1));
     const uint64_t MB = f2s(fmb), LO = f2s(fmb - fqm), HI = f2s(fmb + fqm);
+    uint32_t wd[2 * B];
 #pragma unroll
     for (int c = 0; c < 4; c++) {
-        const uint64_t gc = col_pair(S.colG, t.col(c));
         uint32_t f[16];
 #pragma unroll
         for (int m = 0; m < 8; m++) {
-            // one rounding of the exact product, then the clamp on the biased code
-            uint64_t uu = ffma2(x2[m][c], gc, MB);      // bits: 0x4B400000 | (q + 2^(B-1))
+            // one rounding of the product, then the clamp on the biased code
+            uint64_t uu = ffma2(x2[m][c], g[c], MB);      // bits: 0x4B400000 | (q + 2^(B-1))
             if (CLIP) uu = clamp2r(uu, LO, HI);
             f[2 * m] = (uint32_t)uu;
             f[2 * m + 1] = (uint32_t)(uu >> 32);
         }
-        uint32_t wd[8];
-        pack_codes<B>(f, wd);
-        store_chunk<B>(page + chunk_off<B>(t.w, t.col(c)), wd);
+        pack_codes<B>(f, wd, c);
     }
+    store_block<B>(block_ptr<B>(page, t.tid), wd);
 }
 
 // ---------------------------------------------------------------- the fit
 // Key-Row-Aware Dual-axis Fitting of the register tile (Sec. 4.3, App. C.1)
 // and packing into the page (App. C.3 step 6). The tile holds Z with
 // X_ij = a_i Z_ij (a_i > 0 a per-row factor: a_i = alpha r_i in the decode
-// step, 1 when packing a dense state, S.rA holds it when `scaled`); rs[r] holds
-// the partial sums of |Z| of the thread's rows over its 4 columns. Readout
-// partials (y_part), when given, ride on the column-start round and are summed
-// by threads 128..255 while threads 0..127 derive the start. On return the page holds r, c and the
-// codes. Requires the old page to be fully consumed by every thread and
-// S.colM zeroed before the previous CTA barrier.
-template <int B>
+// step, 1 when packing a dense state, S.rA holds it when `scaled`); rs[r]
+// holds the partial sums of |Z| of the thread's rows over its 4 columns.
+// `between` runs once the row partials are in shared memory, while threads
+// 0..127 derive the row factors (the producer refills a stage there). On
+// return the page holds r, c and the codes. Requires every thread to be done
+// reading the old page.
+template <int B, class Between>
 __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *page, const float *w2v,
                                          const float *wisv, bool scaled, uint64_t (&x2)[8][4],
-                                         float (&rs)[16], const float (&y_part)[4], bool with_y,
-                                         float *y_out, int fit_iters) {
+                                         const float (&rs)[16], int fit_iters, const Between &between) {
     constexpr int qm = (1 << (B - 1)) - 1;
     constexpr float fqm = (float)qm;
-    const float mu = __frcp_rn(fqm);
     uint16_t *page_r = (uint16_t *)page;
     uint16_t *page_c = (uint16_t *)(page + 256);
-    // Row factors r_i = m_i^(1/2) w_i^(-1/2), m_i = (1/128) sum_j |X_ij|.
+    // Row factors r_i = m_i^(1/2) w_i^(-1/2), m_i = (1/128) sum_j |X_ij|: the
+    // band's 4 lanes reduce-scatter their partials, the 8 warps' sums meet in
+    // shared memory.
     {
-        int rr;
-        const float sz = warp_row_sums(rs, t.l, rr);
-        const int i = t.row(rr);
-        const float a = scaled ? S.rA[i] : 1.f;
+        float part[4];
+        row_sum_scatter(rs, t.cg, part);
+        *(float4 *)&S.red[t.w * 128 + t.row(8 * (t.cg & 1) + 4 * (t.cg >> 1))] =
+            make_float4(part[0], part[1], part[2], part[3]);
+    }
+    __syncthreads();
+    between();
+    if (t.tid < 128) {
+        const int i = t.tid;
+        float sz = 0.f;
+#pragma unroll
+        for (int wv = 0; wv < 8; wv++) sz += S.red[wv * 128 + i];
+        const float a = scaled ? S.rA[prow(i)] : 1.f;
         const float m = (a * sz) * (1.0f / 128.0f);
         const float rf = __half2float(__float2half_rn(
             fminf(fmaxf(__fmul_rn(sqrtf(m), wisv[i]), kF16Min), kF16Max)));
-        if ((t.l & 1) == 0) {
-            S.rRho[i] = __frcp_rn(rf) * a;                 // X' = rho_i X = (rho_i a_i) Z
-            S.rAl[i] = w2v[i] * (rf * rf);                 // w_i^2 r_i^2
-            page_r[i] = f16_bits(rf);
-        }
+        S.rRho[prow(i)] = __frcp_rn(rf) * a;              // X' = rho_i X = (rho_i a_i) Z
+        S.rAl[prow(i)] = w2v[i] * (rf * rf);              // w_i^2 r_i^2
+        page_r[i] = f16_bits(rf);
     }
-    __syncwarp();
-    // X' = X rho_i (row-normalised state) and the clip-free column start,
-    // max_i |X'_ij| merged across warps by an atomic max on the (non-negative)
-    // float bits: exact and order-free.
+    __syncthreads();
+    // X' = X rho_i (row-normalised state) and the clip-free column start
+    // c0_j = max_i |X'_ij| / qmax, reduced inside the warp.
     float cm[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int p = 0; p < 4; p++) {
@@ -351,128 +365,90 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
             cm[c] = fmax3(cm[c], fabsf(f2lo(x2[2 * p + 1][c])), fabsf(f2hi(x2[2 * p + 1][c])));
         }
     }
-#pragma unroll
-    for (int c = 0; c < 4; c++) atomicMax(&S.colM[t.col(c)], __float_as_uint(cm[c]));
-    if (with_y) {
-        const float v[1][4] = {{y_part[0], y_part[1], y_part[2], y_part[3]}};
-        cols_to_red<1>(t, S.red, 2, v);
-    }
-    if (t.tid == 0) {
-        S.flags[1] = 0;
-        S.flags[2] = 0;
-    }
-    __syncthreads();
-    // Column start (threads 0..127, one column each) beside the readout sums
-    // (threads 128..255).
-    if (t.tid < 128) {
-        const float mx = __uint_as_float(S.colM[t.tid]);
-        const float c0 = __fmul_rn(mx, mu);
-        if (c0 > kF16Max) S.flags[1] = 1;                 // start capped: codes may clip
-        const float cc = fminf(fmaxf(c0, kF16Min), kF16Max);
-        const float gi = __frcp_rn(cc);
-        S.colC[t.tid] = cc;
-        S.colX[t.tid] = mx;
-        S.colG[t.tid] = make_float2(gi, gi);
-    } else if (with_y) {
-        const int j = t.tid - 128;
-        float s = S.red[(2 * 8) * 128 + j];
-#pragma unroll
-        for (int wv = 1; wv < 8; wv++) s += S.red[(2 * 8 + wv) * 128 + j];
-        y_out[j] = s;
-    }
-    __syncthreads();
-    const bool clip0 = S.flags[1] != 0;
+    // this lane's column (own_col): its max, its current scale, its reciprocal
+    const float mx = col_max_scatter(cm, t.rg);
+    const float c0 = __fmul_rn(mx, __frcp_rn(fqm));
+    const bool clip0 = __any_sync(0xffffffffu, c0 > kF16Max);   // start capped: codes may clip
+    float cc = fminf(fmaxf(c0, kF16Min), kF16Max);
+    float gi = __frcp_rn(cc);
     uint64_t g[4];
 #pragma unroll
-    for (int c = 0; c < 4; c++) g[c] = col_pair(S.colG, t.col(c));
+    for (int c = 0; c < 4; c++) g[c] = f2s(col_gather(gi, t, c));
     // Fixed-code least-squares updates: c_j = sum alpha_i q_ij X'_ij / sum alpha_i q_ij^2
     // (alpha_i = w_i^2 r_i^2: the w^2-weighted objective in the X' domain).
+    bool clip = clip0;
     for (int it = 0; it < fit_iters; it++) {
-        const bool clip = it > 0 || clip0;
-        if (it > 0) {
-#pragma unroll
-            for (int c = 0; c < 4; c++) g[c] = col_pair(S.colG, t.col(c));
-        }
         uint64_t n[4] = {0, 0, 0, 0}, d[4] = {0, 0, 0, 0};
-        // the clip decision is per tile: one branch here, none per element
-        if (clip) ls_sums<B, true>(t, S, x2, g, n, d);
+        // the clip decision is per warp: one branch here, none per element
+        if (it > 0 || clip0) ls_sums<B, true>(t, S, x2, g, n, d);
         else ls_sums<B, false>(t, S, x2, g, n, d);
-        {
-            const float v[2][4] = {{pair_sum(n[0]), pair_sum(n[1]), pair_sum(n[2]), pair_sum(n[3])},
-                                   {pair_sum(d[0]), pair_sum(d[1]), pair_sum(d[2]), pair_sum(d[3])}};
-            cols_to_red<2>(t, S.red, 0, v);
+        const float nv[4] = {pair_sum(n[0]), pair_sum(n[1]), pair_sum(n[2]), pair_sum(n[3])};
+        const float dv[4] = {pair_sum(d[0]), pair_sum(d[1]), pair_sum(d[2]), pair_sum(d[3])};
+        float num, den;
+        col_sum2_scatter(nv, dv, t.rg, num, den);
+        // num and den carry fp32 summation error already; a 2-ulp quotient adds nothing
+        if (den > 0.f) cc = fminf(fmaxf(__fdividef(num, den), kF16Min), kF16Max);
+        if (it + 1 < fit_iters) {
+            gi = __frcp_rn(cc);
+        } else {
+            // storage precision of c; codes can clip only where max |X'| / c >= qmax + 1/2
+            const float cf = __half2float(__float2half_rn(cc));
+            gi = __frcp_rn(cf);
+            if ((t.rg & 1) == 0) page_c[t.own_col()] = f16_bits(cf);
+            clip = __any_sync(0xffffffffu, __fmul_rn(mx, gi) >= fqm + 0.5f);
         }
-        __syncthreads();
-        if (t.tid < 128) {
-            float num = 0.f, den = 0.f;
 #pragma unroll
-            for (int wv = 0; wv < 8; wv++) {
-                num += S.red[wv * 128 + t.tid];
-                den += S.red[(8 + wv) * 128 + t.tid];
-            }
-            // num and den carry fp32 summation error already; a 2-ulp quotient adds nothing
-            float c = S.colC[t.tid];
-            if (den > 0.f) c = fminf(fmaxf(__fdividef(num, den), kF16Min), kF16Max);
-            if (it + 1 < fit_iters) {
-                S.colC[t.tid] = c;
-                const float gi = __frcp_rn(c);
-                S.colG[t.tid] = make_float2(gi, gi);
-            } else {
-                // storage precision of c; codes can clip only where max |X'| / c >= qmax + 1/2
-                const float cf = __half2float(__float2half_rn(c));
-                const float gi = __frcp_rn(cf);
-                page_c[t.tid] = f16_bits(cf);
-                S.colG[t.tid] = make_float2(gi, gi);
-                if (__fmul_rn(S.colX[t.tid], gi) >= fqm + 0.5f) S.flags[2] = 1;
-            }
-        }
-        __syncthreads();
+        for (int c = 0; c < 4; c++) g[c] = f2s(col_gather(gi, t, c));
     }
     // Final codes with the stored scales.
-    const bool clip = S.flags[2] != 0;
-    if (clip) final_codes<B, true>(t, S, page, x2);
-    else final_codes<B, false>(t, S, page, x2);
+    if (clip) final_codes<B, true>(t, page, x2, g);
+    else final_codes<B, false>(t, page, x2, g);
 }
 
-// FP16 pivot head: store fp16(a_i Z) (saturating) in band-major order; a row
-// pair is one 32-bit word of the chunk.
+// FP16 pivot head: store fp16(a_i Z) (saturating) in the chunk order; a row
+// pair is one 32-bit word of a chunk.
 __device__ __forceinline__ void pack_pivot(const T &t, uint8_t *page, const uint64_t (&x2)[8][4],
                                            float a) {
+    uint32_t wd[2 * kPivot];
 #pragma unroll
-    for (int c = 0; c < 4; c++) {
-        uint32_t wd[8];
+    for (int c = 0; c < 4; c++)
 #pragma unroll
         for (int m = 0; m < 8; m++)
-            wd[m] = (uint32_t)f16_bits(f16_round_sat(a * f2lo(x2[m][c]))) |
-                    ((uint32_t)f16_bits(f16_round_sat(a * f2hi(x2[m][c]))) << 16);
-        store_chunk<kPivot>(page + chunk_off<kPivot>(t.w, t.col(c)), wd);
-    }
+            wd[8 * c + m] = (uint32_t)f16_bits(f16_round_sat(a * f2lo(x2[m][c]))) |
+                            ((uint32_t)f16_bits(f16_round_sat(a * f2hi(x2[m][c]))) << 16);
+    store_block<kPivot>(block_ptr<kPivot>(page, t.tid), wd);
 }
 
 // Reconstruct the column-scaled codes c_j q_ij (exact in fp32) or the FP16
 // values of a pivot head; the row factor stays separate.
 template <int B>
 __device__ __forceinline__ void load_tile(const T &t, const uint8_t *page, uint64_t (&x2)[8][4]) {
-    const uint16_t *page_c = (const uint16_t *)(page + 256);
+    uint32_t wd[2 * B];
+    load_block<B>(block_ptr<B>((uint8_t *)page, t.tid), wd);
+    if constexpr (B == kPivot) {
 #pragma unroll
-    for (int c = 0; c < 4; c++) {
-        uint32_t wd[8];
-        load_chunk<B>(page + chunk_off<B>(t.w, t.col(c)), wd);
-        if (B == kPivot) {
+        for (int c = 0; c < 4; c++)
 #pragma unroll
             for (int m = 0; m < 8; m++)
-                x2[m][c] = f2(f16_val((uint16_t)(wd[m] & 0xFFFFu)), f16_val((uint16_t)(wd[m] >> 16)));
-        } else {
-            // f = 1.5*2^23 + u s (s = 1 or the pair's high scale): fma(f, c/s, -1.5*2^23 c/s)
-            // = c u exactly (c fp16 and normal, u < 2^8: 19 significant bits; the
-            // offset has 12), and c u - c 2^(B-1) = c q is exact as well.
-            const uint64_t cj = f2s(f16_val(page_c[t.col(c)]));
-            const uint64_t cc = fmul2(cj, f2(1.0f, hi_scale<B>()));
-            const uint64_t oc = fmul2(cc, f2s(-kMagic));
-            const uint64_t bc = fmul2(cj, f2s(-(float)(1 << (B - 1))));
+                x2[m][c] = f2(f16_val((uint16_t)(wd[8 * c + m] & 0xFFFFu)), f16_val((uint16_t)(wd[8 * c + m] >> 16)));
+        return;
+    } else {
+    // the thread's 4 column scales: one 8-byte load
+    const uint2 c4 = *(const uint2 *)(page + 256 + 2 * t.col(0));
+    const uint16_t ch[4] = {(uint16_t)(c4.x & 0xFFFFu), (uint16_t)(c4.x >> 16), (uint16_t)(c4.y & 0xFFFFu),
+                            (uint16_t)(c4.y >> 16)};
 #pragma unroll
-            for (int m = 0; m < 8; m++) x2[m][c] = fadd2(ffma2(code_pair<B>(wd, m), cc, oc), bc);
-        }
+    for (int c = 0; c < 4; c++) {
+        // f = 1.5*2^23 + u s (s = 1 or the pair's high scale): fma(f, c/s, -1.5*2^23 c/s)
+        // = c u exactly (c fp16 and normal, u < 2^8: 19 significant bits; the
+        // offset has 12), and c u - c 2^(B-1) = c q is exact as well.
+        const uint64_t cj = f2s(f16_val(ch[c]));
+        const uint64_t cc = fmul2(cj, f2(1.0f, hi_scale<B>()));
+        const uint64_t oc = fmul2(cc, f2s(-kMagic));
+        const uint64_t bc = fmul2(cj, f2s(-(float)(1 << (B - 1))));
+#pragma unroll
+        for (int m = 0; m < 8; m++) x2[m][c] = fadd2(ffma2(code_pair<B>(wd, c, m), cc, oc), bc);
+    }
     }
 }
 
@@ -499,9 +475,9 @@ struct DecodeArgs {
     int fit_iters;
 };
 
-// Producer: start the copies of the item (head h, batch entry b, a valid slot)
-// into stage s. The writeback loads delta into the v slot and needs no q; the
-// readout needs no w2, wis.
+// Producer warp: start the copies of the item (head h, batch entry b, a valid
+// slot) into stage s. The writeback loads delta into the v slot and needs no
+// q; the readout needs no w2, wis.
 template <int MODE>
 __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h, int b, int slot, int s,
                                       int lane) {
@@ -532,8 +508,8 @@ __device__ __forceinline__ void issue(const DecodeArgs &a, const Smem &S, int h,
 // One decode step of one head page staged in shared memory (width B).
 // `ok` is this thread's verdict on the stage's copies; the first CTA barrier
 // takes the OR of the negations, and on a stalled copy every thread returns
-// false there (what it read before is discarded). `refill` runs after that
-// barrier; the page itself is rewritten in place afterwards.
+// false there (what it read before is discarded). `refill` runs once per item,
+// after that barrier; the page itself is rewritten in place afterwards.
 //
 // With a_i = alpha r_i (> 0) and Z_ij = c_j q_ij + (beta k_i / a_i) delta_j the
 // update is X_ij = a_i Z_ij: one fma per element instead of two.
@@ -547,51 +523,29 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
                                             float beta, float *y_out, float *delta_out, int fit_iters,
                                             bool ok, const Refill &refill) {
     const uint16_t *page_r = (const uint16_t *)st.page;
-    // Row constants of the warp's band (warp-local).
-    if (t.l < 16) {
-        const int i = t.row(t.l);
+    // Row constants (threads 0..127, one row each).
+    if (t.tid < 128) {
+        const int i = t.tid, pi = prow(i);
         const float a = fmaxf(B == kPivot ? alpha : alpha * f16_val(page_r[i]), 1e-30f);
         const float ki = st.k[i];
-        S.rKap[i] = ki * a;
-        S.rBkp[i] = __fdividef(beta * ki, a);          // within 2 ulp: Z carries rounding anyway
-        if (MODE != kWriteback) S.rQa[i] = st.q[i] * a;
-        S.rA[i] = a;
+        S.rKap[pi] = ki * a;
+        S.rBkp[pi] = __fdividef(beta * ki, a);          // within 2 ulp: Z carries rounding anyway
+        if (MODE != kWriteback) S.rQa[pi] = st.q[i] * a;
+        S.rA[pi] = a;
     }
-    if (MODE != kReadout && t.tid < 128) S.colM[t.tid] = 0u;
     uint64_t x2[8][4];
     load_tile<B>(t, st.page, x2);
-    __syncwarp();
+    if (__syncthreads_or(!ok)) return false;
+    const bool fit = MODE != kReadout && B != kPivot;
+    if (!fit) refill();
+    uint64_t dl[4];
     if constexpr (MODE == kWriteback) {
-        if (__syncthreads_or(!ok)) return false;
-        refill();
-        // Z = c q + (beta k / a) delta with the readout's delta; row sums of |Z|.
-        uint64_t dl[4];
-#pragma unroll
-        for (int c = 0; c < 4; c++) dl[c] = f2s(st.v[t.col(c)]);
-        float rs[16];
-#pragma unroll
-        for (int p = 0; p < 4; p++) {
-            uint64_t blo, bhi;
-            row_pairs(S.rBkp, t, p, blo, bhi);
-#pragma unroll
-            for (int c = 0; c < 4; c++) {
-                x2[2 * p][c] = ffma2(blo, dl[c], x2[2 * p][c]);
-                x2[2 * p + 1][c] = ffma2(bhi, dl[c], x2[2 * p + 1][c]);
-            }
-            abs_row_sums(x2[2 * p], rs[4 * p], rs[4 * p + 1]);
-            abs_row_sums(x2[2 * p + 1], rs[4 * p + 2], rs[4 * p + 3]);
-        }
-        if (B == kPivot) {
-            pack_pivot(t, st.page, x2, fmaxf(alpha, 1e-30f));
-            return true;
-        }
-        const float none[4] = {0.f, 0.f, 0.f, 0.f};
-        fit_pack<B>(t, S, st.page, st.w2, st.wis, true, x2, rs, none, false, nullptr, fit_iters);
-        return true;
-    }
-    // Step 2a: retrieval u_j = sum_i k_i a_i (c_j q_ij).
-    {
-        uint64_t ua[4] = {0, 0, 0, 0};              // one accumulator per column: fewer live registers
+        const float4 d4 = *(const float4 *)&st.v[t.col(0)];
+        dl[0] = f2s(d4.x); dl[1] = f2s(d4.y); dl[2] = f2s(d4.z); dl[3] = f2s(d4.w);
+    } else {
+        // Step 2a: retrieval u_j = sum_i k_i a_i (c_j q_ij), reduced over the
+        // column group; delta_j = v_j - u_j for the lane's column, gathered.
+        uint64_t ua[4] = {0, 0, 0, 0};
 #pragma unroll
         for (int p = 0; p < 4; p++) {
             uint64_t klo, khi;
@@ -602,64 +556,50 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
                 ua[c] = ffma2(khi, x2[2 * p + 1][c], ua[c]);
             }
         }
-        const float v[1][4] = {{pair_sum(ua[0]), pair_sum(ua[1]), pair_sum(ua[2]), pair_sum(ua[3])}};
-        cols_to_red<1>(t, S.red, 0, v);
-    }
-    if (__syncthreads_or(!ok)) return false;
-    if (t.tid < 128) {
-        float s = 0.f;
+        const float u4[4] = {pair_sum(ua[0]), pair_sum(ua[1]), pair_sum(ua[2]), pair_sum(ua[3])};
+        const float u = col_sum_scatter(u4, t.rg);
+        const float dj = st.v[t.own_col()] - u;             // delta_j = v_j - u_j
+        if (MODE == kReadout && (t.rg & 1) == 0) delta_out[t.own_col()] = dj;
 #pragma unroll
-        for (int wv = 0; wv < 8; wv++) s += S.red[wv * 128 + t.tid];
-        const float dl = st.v[t.tid] - s;                  // delta_j = v_j - u_j
-        S.colD[t.tid] = make_float2(dl, dl);
-        if (MODE == kReadout) delta_out[t.tid] = dl;
+        for (int c = 0; c < 4; c++) dl[c] = f2s(col_gather(dj, t, c));
     }
-    refill();
-    __syncthreads();
     // Step 2b-3: Z = c q + (beta k / a) delta; readout partials q_i a_i Z_ij.
-    uint64_t dl[4];
-#pragma unroll
-    for (int c = 0; c < 4; c++) dl[c] = col_pair(S.colD, t.col(c));
-    uint64_t ya[4] = {0, 0, 0, 0};                  // one accumulator per column
-    float rs[16];
+    uint64_t ya[4] = {0, 0, 0, 0};
 #pragma unroll
     for (int p = 0; p < 4; p++) {
-        uint64_t blo, bhi, qlo, qhi;
+        uint64_t blo, bhi;
         row_pairs(S.rBkp, t, p, blo, bhi);
-        row_pairs(S.rQa, t, p, qlo, qhi);
 #pragma unroll
         for (int c = 0; c < 4; c++) {
             x2[2 * p][c] = ffma2(blo, dl[c], x2[2 * p][c]);
             x2[2 * p + 1][c] = ffma2(bhi, dl[c], x2[2 * p + 1][c]);
-            ya[c] = ffma2(qlo, x2[2 * p][c], ya[c]);
-            ya[c] = ffma2(qhi, x2[2 * p + 1][c], ya[c]);
+        }
+        if (MODE != kWriteback) {
+            uint64_t qlo, qhi;
+            row_pairs(S.rQa, t, p, qlo, qhi);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                ya[c] = ffma2(qlo, x2[2 * p][c], ya[c]);
+                ya[c] = ffma2(qhi, x2[2 * p + 1][c], ya[c]);
+            }
         }
     }
-    const float yp[4] = {pair_sum(ya[0]), pair_sum(ya[1]), pair_sum(ya[2]), pair_sum(ya[3])};
-    // row sums of |Z| once the readout accumulators are reduced (fewer live registers)
-    if (MODE == kFused) {
-#pragma unroll
-        for (int p = 0; p < 4; p++) {
-            abs_row_sums(x2[2 * p], rs[4 * p], rs[4 * p + 1]);
-            abs_row_sums(x2[2 * p + 1], rs[4 * p + 2], rs[4 * p + 3]);
-        }
+    if (MODE != kWriteback) {
+        const float y4[4] = {pair_sum(ya[0]), pair_sum(ya[1]), pair_sum(ya[2]), pair_sum(ya[3])};
+        const float yj = col_sum_scatter(y4, t.rg);
+        if ((t.rg & 1) == 0) y_out[t.own_col()] = yj;
     }
-    if (B == kPivot || MODE == kReadout) {
-        const float v[1][4] = {{yp[0], yp[1], yp[2], yp[3]}};
-        cols_to_red<1>(t, S.red, 2, v);
-        __syncthreads();
-        if (t.l < 16) {
-            const int j = 16 * t.w + t.l;
-            float s = S.red[(2 * 8) * 128 + j];
-#pragma unroll
-            for (int wv = 1; wv < 8; wv++) s += S.red[(2 * 8 + wv) * 128 + j];
-            y_out[j] = s;
-        }
-        if (MODE == kFused) pack_pivot(t, st.page, x2, fmaxf(alpha, 1e-30f));
+    if (MODE == kReadout) return true;
+    if (B == kPivot) {
+        pack_pivot(t, st.page, x2, fmaxf(alpha, 1e-30f));
         return true;
     }
     // Steps 4-6: refit and repack in place.
-    fit_pack<B>(t, S, st.page, st.w2, st.wis, true, x2, rs, yp, true, y_out, fit_iters);
+    float rs[16];
+#pragma unroll
+    for (int m = 0; m < 8; m++) abs_row_sums(x2[m], rs[2 * m], rs[2 * m + 1]);
+    if constexpr (B != kPivot)
+        fit_pack<B>(t, S, st.page, st.w2, st.wis, true, x2, rs, fit_iters, refill);
     return true;
 }
 
@@ -731,17 +671,19 @@ __device__ __forceinline__ void quantize_item(const T &t, const Smem &S, uint8_t
     float rs[16];
 #pragma unroll
     for (int m = 0; m < 8; m++) {
-        const float *r0 = X + t.row(2 * m) * 128, *r1 = r0 + 128;
-#pragma unroll
-        for (int c = 0; c < 4; c++) x2[m][c] = f2(r0[t.col(c)], r1[t.col(c)]);
+        const float4 r0 = *(const float4 *)(X + t.row(2 * m) * 128 + t.col(0));
+        const float4 r1 = *(const float4 *)(X + t.row(2 * m + 1) * 128 + t.col(0));
+        x2[m][0] = f2(r0.x, r1.x);
+        x2[m][1] = f2(r0.y, r1.y);
+        x2[m][2] = f2(r0.z, r1.z);
+        x2[m][3] = f2(r0.w, r1.w);
         abs_row_sums(x2[m], rs[2 * m], rs[2 * m + 1]);
     }
-    if (B == kPivot) {
+    if constexpr (B == kPivot) {
         pack_pivot(t, page, x2, 1.f);
-        return;
+    } else {
+        fit_pack<B>(t, S, page, w2, wis, false, x2, rs, fit_iters, [] {});
     }
-    const float none[4] = {0.f, 0.f, 0.f, 0.f};
-    fit_pack<B>(t, S, page, w2, wis, false, x2, rs, none, false, nullptr, fit_iters);
 }
 
 __global__ void __launch_bounds__(kThreads, 2) quantize_heads_kernel(PoolArgs a) {
@@ -759,7 +701,6 @@ __global__ void __launch_bounds__(kThreads, 2) quantize_heads_kernel(PoolArgs a)
     if (t.tid < 128) {
         w2[t.tid] = a.tab.w2[h * 128 + t.tid];
         wis[t.tid] = a.tab.wis[h * 128 + t.tid];
-        S.colM[t.tid] = 0u;
     }
     __syncthreads();
     const float *X = a.states + (size_t)b * a.state_stride_b + (size_t)h * kN;
@@ -783,15 +724,13 @@ __device__ __forceinline__ void dequantize_item(const T &t, const uint8_t *page,
     const uint16_t *page_r = (const uint16_t *)page;
 #pragma unroll
     for (int m = 0; m < 8; m++) {
-        float *r0 = out + t.row(2 * m) * 128, *r1 = r0 + 128;
         // r_i c_j z_ij rounded once: c_j q_ij is exact in fp32 (fp16 x 8 bits)
         const uint64_t rr = B == kPivot ? 0 : f2(f16_val(page_r[t.row(2 * m)]), f16_val(page_r[t.row(2 * m + 1)]));
+        uint64_t v[4];
 #pragma unroll
-        for (int c = 0; c < 4; c++) {
-            const uint64_t v = B == kPivot ? x2[m][c] : fmul2(rr, x2[m][c]);
-            r0[t.col(c)] = f2lo(v);
-            r1[t.col(c)] = f2hi(v);
-        }
+        for (int c = 0; c < 4; c++) v[c] = B == kPivot ? x2[m][c] : fmul2(rr, x2[m][c]);
+        *(float4 *)(out + t.row(2 * m) * 128 + t.col(0)) = make_float4(f2lo(v[0]), f2lo(v[1]), f2lo(v[2]), f2lo(v[3]));
+        *(float4 *)(out + t.row(2 * m + 1) * 128 + t.col(0)) = make_float4(f2hi(v[0]), f2hi(v[1]), f2hi(v[2]), f2hi(v[3]));
     }
 }
 

@@ -86,16 +86,17 @@ def test_pivot_head_is_fp16(oracle, rng):
     rb = np.full(D, PIV, np.int8)
     page = oracle.encode_head(X, HEAD, rb, _w(rng))
     assert page.size == D * D * 2
-    # band-major: [band w][column j][row 16w + r]
-    vals = page.view(np.float16).reshape(8, D, 16).transpose(0, 2, 1).reshape(D, D)
+    # chunks [column group t][band g][column 4t + c][row 16g + r]
+    vals = page.view(np.float16).reshape(32, 8, 4, 16).transpose(1, 3, 0, 2).reshape(D, D)
     ref = np.float16(np.clip(X, -65504, 65504))
     assert np.array_equal(vals.astype(np.float64), ref.astype(np.float64))
 
 
 @pytest.mark.parametrize("b", [2, 4, 6, 8])
 def test_bit_layout_with_independent_unpacker(oracle, rng, b):
-    """Head units: offset-binary codes u = q + 2^(b-1), LSB-first, in band-major
-    chunks (band w of 16 rows, column j: the 16 codes of rows 16w..16w+15)."""
+    """Head units: offset-binary codes u = q + 2^(b-1), LSB-first, in chunks of
+    the 16 codes of one band of rows (16g..16g+15) in one column, ordered by
+    column group (4 columns), band, column within the group."""
     X = _state(rng)
     rb = np.full(D, b, np.int8)
     page = oracle.encode_head(X, HEAD, rb, _w(rng))
@@ -104,8 +105,8 @@ def test_bit_layout_with_independent_unpacker(oracle, rng, b):
     assert np.array_equal(page[:256].view(np.uint16), r16)
     assert np.array_equal(page[256:512].view(np.uint16), c16)
     bits = np.unpackbits(page[512:].reshape(8 * D, 2 * b), axis=1, bitorder="little")
-    u = (bits.reshape(8, D, 16, b) * (1 << np.arange(b))).sum(-1)     # [band][col][row in band]
-    u = u.transpose(0, 2, 1).reshape(D, D)
+    u = (bits.reshape(32, 8, 4, 16, b) * (1 << np.arange(b))).sum(-1)   # [group][band][c][row in band]
+    u = u.transpose(1, 3, 0, 2).reshape(D, D)
     assert np.array_equal(u - 2 ** (b - 1), codes.astype(np.int64))
     assert u.min() >= 1
 

@@ -131,8 +131,8 @@ MUTANTS = [
      "        if ((u >> (b - 1 - t)) & 1u)\n            row[p >> 3] |="),
     ("rows_stored_ascending", "codec.c", "        if (rb[t] > b || (rb[t] == b && t < i))",
      "        if (rb[t] < b || (rb[t] == b && t < i))"),
-    ("band_of_row", "codec.c", "        size_t chunk = (size_t)(i / 16) * OR_D + (size_t)j;        /* band-major chunks */",
-     "        size_t chunk = (size_t)(i % 8) * OR_D + (size_t)j;        /* band-major chunks */"),
+    ("band_of_row", "codec.c", "        size_t chunk = ((size_t)(j / 4) * 8 + (size_t)(i / 16)) * 4 + (size_t)(j % 4);",
+     "        size_t chunk = ((size_t)(j / 4) * 8 + (size_t)(i % 8)) * 4 + (size_t)(j % 4);"),
     ("fp16_subnormal_scale", "numerics.c", "        return s | (uint16_t)(a / ldexp(1.0, -24));   /* subnormal: fraction counts 2^-24 */",
      "        return s | (uint16_t)(a / ldexp(1.0, -23));   /* subnormal: fraction counts 2^-24 */"),
     ("row_pivot_risk_without_fp16", "plan.c",
