@@ -39,43 +39,60 @@ def _peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    """nvidia-smi clocks and throttle reasons, sampled every 100 ms by one
+    nvidia-smi process that runs across every timed region."""
     FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap")
 
     def __init__(self, index: int):
         self.index = index
-        self.rows = []
-        self._stop = threading.Event()
-        self._t = None
+        self.proc = None
 
     def start(self):
-        def run():
-            while not self._stop.is_set():
-                try:
-                    out = subprocess.run(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
-                                          "--format=csv,noheader,nounits"], capture_output=True,
-                                         text=True, timeout=5).stdout.strip()
-                    if out:
-                        self.rows.append([x.strip() for x in out.split(",")])
-                except Exception:
-                    pass
-                self._stop.wait(0.2)
-        self._t = threading.Thread(target=run, daemon=True)
-        self._t.start()
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
 
     def stop(self):
-        self._stop.set()
-        if self._t:
-            self._t.join(timeout=10)
-        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
-        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        rows = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=10)
+            except Exception:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            rows = [[x.strip() for x in line.split(",")] for line in out.splitlines() if line.strip()]
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in rows if len(r) > 1 and r[1].replace(".", "").isdigit()]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[k] for r in self.rows for k in range(4)
+        reasons = sorted({names[k] for r in rows for k in range(4)
                           if len(r) > 3 + k and r[3 + k].lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None,
-                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(self.rows)}
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+def _cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine type)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.machine()
 
 
 def _recorded_traffic(units_per_launch: int):
@@ -138,8 +155,89 @@ def cpu_baseline(wl, units: int, min_seconds: float = 10.0):
         done += B * wl.hv
         step += 1
     return {"value": done / elapsed, "unit": UNIT, "cores": O.num_threads(), "kind": "oracle",
+            "cpu_model": _cpu_model(),
             "sample": f"{step} decode steps of one layer for {B} slots x {wl.hv} heads "
                       f"({done} head updates) of the {wl.name} workload, {elapsed:.1f} s"}
+
+
+def secondary_channel(args, dev, peak, _unused=None):
+    """The channel-gate decode workload (one layer of 32 heads with per-key-channel
+    gates, 256 slots, STEPQuant at 4 bits: row units) beside the FP32-state and
+    INT8 rowwise kernels on the same inputs. Its pool is smaller than L2, so a
+    256 MiB buffer is written between timed launches and only the launches are
+    timed (CUDA events around each)."""
+    import torch
+    import paper_2609_38169_gb300 as P
+    from paper_2609_38169_gb300 import workloads as W
+    wl = W.WORKLOADS["channel"]
+    cfg = P.Config.from_workload(wl)
+    Hv, Hk, B = wl.hv, wl.hk, wl.batch
+    st = P.calibrate(cfg, wl, device=dev, steps=min(args.calib_steps, wl.calib_steps), device_inputs=True)
+    plan = P.stepq_fit_scales(cfg, st.omega, st.mean_log_ret, st.dist, st.pivot)
+    mp_dev = W.model_params_torch(W.model_params(wl), dev)
+    fp32_pool = torch.zeros((wl.pool_slots, 1, Hv, 128, 128), dtype=torch.float32, device=dev)
+    all_slots = torch.arange(wl.pool_slots, dtype=torch.int32, device=dev)
+    y = torch.empty((B, Hv, 128), dtype=torch.float32, device=dev)
+    for t in range(wl.warmup_steps):
+        q, k, v, beta, gate = W.torch_step_inputs(wl, mp_dev, t, 0, dev, W.STREAM_WARMUP, batch=wl.pool_slots)
+        P.stepq_fp32_decode_step(cfg, 0, fp32_pool, all_slots, q, k, v, beta, gate, y)
+    pool = P.alloc_pool(plan, wl.pool_slots, dev)
+    P.stepq_quantize_pool(plan, 0, fp32_pool, all_slots, pool)
+    i8_stride = P.stepq_intb_slot_bytes(cfg, 8)
+    i8_pool = torch.zeros(wl.pool_slots * i8_stride, dtype=torch.uint8, device=dev)
+    P.stepq_intb_quantize_pool(cfg, 8, 0, fp32_pool, all_slots, i8_pool)
+    slots = torch.from_numpy(W.slot_permutation(wl)).to(dev)
+    inputs = [W.torch_step_inputs(wl, mp_dev, 1000 + s, 0, dev) for s in range(2)]
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def timed(call, steps, warmup):
+        for s in range(warmup):
+            call(*inputs[s % 2])
+        torch.cuda.synchronize(dev)
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(steps)]
+        for s in range(steps):
+            flush.fill_(s & 0xFF)                         # L2 holds none of the pool
+            evs[s][0].record(stream)
+            call(*inputs[s % 2])
+            evs[s][1].record(stream)
+        torch.cuda.synchronize(dev)
+        return [a.elapsed_time(b) for a, b in evs]
+
+    steps = max(args.steps, 10)
+    ms = timed(lambda q, k, v, beta, gate: P.stepq_decode_step(plan, 0, pool, slots, q, k, v, beta, gate, y,
+                                                                pool_slots=wl.pool_slots), steps, args.warmup)
+    fp_ms = timed(lambda q, k, v, beta, gate: P.stepq_fp32_decode_step(cfg, 0, fp32_pool, slots, q, k, v, beta,
+                                                                        gate, y, pool_slots=wl.pool_slots),
+                  steps, args.warmup)
+    i8_ms = timed(lambda q, k, v, beta, gate: P.stepq_intb_decode_step(cfg, 8, 0, i8_pool, slots, q, k, v, beta,
+                                                                        gate, y, pool_slots=wl.pool_slots),
+                  steps, args.warmup)
+    assert P.stepq_device_error() == 0
+    units = B * Hv
+    io_b = B * (Hk * 2 * 512 + Hv * (512 + 4 + 512 + 512))
+    page_b = int(B * 2 * plan.head_bytes.astype(np.int64).sum())
+    avg = statistics.mean(ms) / 1e3
+    achieved = (page_b + io_b) / avg / 1e9
+    fp_b = units * 2 * 65536 + io_b
+    i8_b = units * 2 * (i8_stride // Hv) + io_b
+    out = {"workload": "channel-wise gate decode: 1 layer x 32 heads, d=128, 256 slots (random permutation), "
+                       "per-key-channel gates, STEPQuant @4 (row units); L2 flushed between launches",
+           "metric": "head-state decode updates/sec (one layer launch)", "unit": UNIT,
+           "value": units / avg, "ms_per_launch": avg * 1e3,
+           "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                        "frac": achieved / peak, "traffic": None, "bytes_per_launch": page_b + io_b,
+                        "avg_launch_us": avg * 1e6},
+           "baselines": {
+               "fp32_state": {"value": units / (statistics.mean(fp_ms) / 1e3), "ms_per_launch": statistics.mean(fp_ms),
+                              "achieved_gbs": fp_b / (statistics.mean(fp_ms) / 1e3) / 1e9},
+               "int8_rowwise": {"value": units / (statistics.mean(i8_ms) / 1e3), "ms_per_launch": statistics.mean(i8_ms),
+                                "achieved_gbs": i8_b / (statistics.mean(i8_ms) / 1e3) / 1e9}},
+           "cpu_baseline": None}
+    if not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(wl, 512, min_seconds=5.0)
+    return out
 
 
 def run_reference(args):
@@ -177,6 +275,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="stepq", choices=["stepq", "reference"])
     ap.add_argument("--no-baselines", action="store_true")
+    ap.add_argument("--no-secondary", action="store_true", help="skip the channel-gate row-unit line")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-units", type=int, default=4096)
     ap.add_argument("--ref-units", type=int, default=1024)
@@ -297,7 +396,6 @@ def main():
     clocks = ClockSampler(dev.index if dev.index is not None else 0)
     clocks.start()
     total_ms, launch_ms = timed(step_stepq, args.steps, args.warmup, per_launch=True, name="stepq_decode")
-    clk = clocks.stop()
     assert P.stepq_device_error() == 0
     units_per_step = L * B * Hv
     total_ms, value = reduce_over_ranks(total_ms, units_per_step * args.steps, world, dev)
@@ -389,9 +487,13 @@ def main():
         step_done[s % (lookahead + 1)].record(stream)
 
     e2e_steps = max(3, args.steps // 2)
-    e2e_ms, _ = timed(step_e2e, e2e_steps, 2, name="stepq_e2e")
-    e2e_ms, e2e_value = reduce_over_ranks(e2e_ms, units_per_step * e2e_steps, world, dev)
-    e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+    # three end-to-end regions; the median is reported (host-side copy scheduling varies)
+    e2e_values = []
+    for rep in range(3):
+        e2e_ms, _ = timed(step_e2e, e2e_steps, 2, name=f"stepq_e2e{rep}")
+        e2e_values.append(reduce_over_ranks(e2e_ms, units_per_step * e2e_steps, world, dev)[1])
+    e2e = {"value": statistics.median(e2e_values), "unit": UNIT, "h2d_bytes_per_step": h2d,
+           "d2h_bytes_per_step": d2h, "regions": e2e_values}
 
     baselines = {}
     if not args.no_baselines:
@@ -408,6 +510,10 @@ def main():
                              "ms_per_step": i8_ms / nb,
                              "achieved_gbs": L * i8_bytes * nb / (i8_ms / 1e3) / 1e9},
         }
+    clk = clocks.stop()
+    secondary = None
+    if not args.no_secondary and world == 1:
+        secondary = secondary_channel(args, dev, peak, None)
 
     if rank == 0:
         cpu = None
@@ -425,6 +531,7 @@ def main():
                        "parallelism": f"replicas x{world}"},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": L * args.steps, "clocks": clk, "baselines": baselines,
+            "secondary": secondary,
             "wall_s": {k: round(v, 4) for k, v in wall_s.items()},
         }
         print(json.dumps(line), flush=True)

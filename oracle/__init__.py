@@ -81,7 +81,7 @@ def _declare(L):
         "or_encode_head": (None, [P, I, P, P, I, P]),
         "or_decode_head": (None, [P, I, P, P]),
         "or_decode_head_f32": (None, [P, I, P, P]),
-        "or_step_head": (None, [P, I, P, P, I, P, P, P, F, P, I, P]),
+        "or_step_head": (None, [P, I, P, P, I, P, P, P, F, P, I, P, P]),
         "or_unpack_head": (None, [P, I, P, P, P, P, P]),
         "or_fit_debug": (None, [P, I, P, P, I, P, P, P]),
         "or_intb_head_bytes": (C.c_size_t, [I]),
@@ -101,7 +101,7 @@ def _declare(L):
         "or_layout": (I, [I, I, I, P, P, P, P]),
         "or_pool_encode": (None, [I, I, P, P, I, P, U64, P, P, I, P]),
         "or_pool_decode": (None, [I, I, P, P, U64, P, P, I, P]),
-        "or_pool_step": (None, [I, I, I, I, P, P, I, P, U64, P, P, I, P, P, P, P, P, P]),
+        "or_pool_step": (None, [I, I, I, I, P, P, I, P, U64, P, P, I, P, P, P, P, P, P, P]),
         "or_pool_step_units": (None, [I, I, I, I, P, P, I, P, U64, P, P, I, P, P, P, P, P, P, P, P]),
         "or_intb_pool_step": (None, [I, I, I, I, U64, U64, P, P, I, P, P, P, P, P, P]),
         "or_calib_observe": (None, [I, I, I, I, P, P, P, P, P, P]),
@@ -269,7 +269,7 @@ def step_head(page, unit_kind, rb, w, q, k, v, beta, gate, fit_iters=1):
     y = np.zeros(D, np.float32)
     lib().or_step_head(_p(page), unit_kind, _p(_i8(rb)), _p(_f32(w)), fit_iters, _p(_f32(q)),
                        _p(_f32(k)), _p(_f32(v)), float(beta), _p(gate), int(gate.size == D),
-                       _p(y))
+                       _p(y), None)
     return page, y
 
 
@@ -457,16 +457,19 @@ def pool_decode(plan: OraclePlan, pool: np.ndarray, layer: int, slots) -> np.nda
     return out
 
 
-def pool_step(plan: OraclePlan, pool: np.ndarray, layer: int, slots, inp) -> np.ndarray:
+def pool_step(plan: OraclePlan, pool: np.ndarray, layer: int, slots, inp, with_delta=False):
+    """One decode step of every (slot, head) of the layer in place; returns y, or
+    (y, delta) with delta_j = v_j - k^T D S_hat (fp64) when asked."""
     slots = np.ascontiguousarray(slots, np.int32)
     B = len(slots)
     y = np.zeros((B, plan.hv, D), np.float32)
+    delta = np.zeros((B, plan.hv, D), np.float64) if with_delta else None
     lib().or_pool_step(plan.unit_kind, plan.hk, plan.hv, int(plan.gate_per_row),
                        _p(plan.layer_row_bits(layer)), _p(plan.layer_w(layer)), plan.fit_iters,
                        _p(plan.layer_head_off(layer)), plan.slot_stride, _p(pool), _p(slots), B,
                        _p(_f32(inp.q)), _p(_f32(inp.k)), _p(_f32(inp.v)), _p(_f32(inp.beta)),
-                       _p(_f32(inp.gate)), _p(y))
-    return y
+                       _p(_f32(inp.gate)), _p(y), _p(delta) if with_delta else None)
+    return (y, delta) if with_delta else y
 
 
 def pool_step_units(plan: OraclePlan, pool, layer, slots, inp, unit_b, unit_h) -> np.ndarray:

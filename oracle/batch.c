@@ -45,7 +45,7 @@ static void step_one(int unit_kind, int Hk, int Hv, int gate_per_row,
                      const int8_t *layer_row_bits, const float *layer_w, int fit_iters,
                      const uint64_t *layer_head_off, uint64_t slot_stride, uint8_t *pool,
                      const int32_t *slots, int b, int h, const float *q, const float *k,
-                     const float *v, const float *beta, const float *gate, float *y)
+                     const float *v, const float *beta, const float *gate, float *y, double *delta)
 {
     int hk = h / (Hv / Hk);
     const float *g = gate_per_row ? gate + ((size_t)b * Hv + h) * OR_D : gate + (size_t)b * Hv + h;
@@ -53,20 +53,20 @@ static void step_one(int unit_kind, int Hk, int Hv, int gate_per_row,
                  layer_row_bits + (size_t)h * OR_D, layer_w + (size_t)h * OR_D, fit_iters,
                  q + ((size_t)b * Hk + hk) * OR_D, k + ((size_t)b * Hk + hk) * OR_D,
                  v + ((size_t)b * Hv + h) * OR_D, beta[(size_t)b * Hv + h], g, gate_per_row,
-                 y + ((size_t)b * Hv + h) * OR_D);
+                 y + ((size_t)b * Hv + h) * OR_D, delta ? delta + ((size_t)b * Hv + h) * OR_D : NULL);
 }
 
 void or_pool_step(int unit_kind, int Hk, int Hv, int gate_per_row, const int8_t *layer_row_bits,
                   const float *layer_w, int fit_iters, const uint64_t *layer_head_off,
                   uint64_t slot_stride, uint8_t *pool, const int32_t *slots, int B,
                   const float *q, const float *k, const float *v, const float *beta,
-                  const float *gate, float *y)
+                  const float *gate, float *y, double *delta)
 {
 #pragma omp parallel for collapse(2) schedule(dynamic)
     for (int b = 0; b < B; b++)
         for (int h = 0; h < Hv; h++)
             step_one(unit_kind, Hk, Hv, gate_per_row, layer_row_bits, layer_w, fit_iters,
-                     layer_head_off, slot_stride, pool, slots, b, h, q, k, v, beta, gate, y);
+                     layer_head_off, slot_stride, pool, slots, b, h, q, k, v, beta, gate, y, delta);
 }
 
 /* Only the listed (batch index, head) units; the rest of the pool is untouched. */
@@ -81,7 +81,7 @@ void or_pool_step_units(int unit_kind, int Hk, int Hv, int gate_per_row,
     for (int t = 0; t < n_units; t++)
         step_one(unit_kind, Hk, Hv, gate_per_row, layer_row_bits, layer_w, fit_iters,
                  layer_head_off, slot_stride, pool, slots, unit_b[t], unit_h[t], q, k, v, beta,
-                 gate, y);
+                 gate, y, NULL);
 }
 
 /* Uniform INT-b pool: head h of the layer at layer_off + h * head_bytes. */

@@ -26,12 +26,13 @@
  *  - codes are stored offset-binary u = q + 2^(b-1), LSB-first per row.
  *
  * Page layout of one head (all pieces 16-byte multiples):
- *   integer head unit: r[128] fp16 | c[128] fp16 | codes in chunks of the 16
- *                      codes of one band of rows (16g..16g+15) in one column
- *                      (2b bytes), ordered by column group (columns 4t..4t+3),
- *                      then band g, then column within the group
- *   pivot head unit:   the same chunk order of fp16 values (32 bytes per
- *                      chunk), no scales
+ *   integer head unit: r[128] fp16 | c[128] fp16 | codes: the 16 codes of one
+ *                      band of rows (16g..16g+15) in one column form a chunk of
+ *                      2b bytes; the four chunks of columns 4t..4t+3 in band g
+ *                      form one stream of 2b words, stored as 16-byte pieces
+ *                      interleaved over the 32 (band, column quad) streams of
+ *                      each group of 16 columns (see bit_addr)
+ *   pivot head unit:   the same arrangement of fp16 values (b = 16), no scales
  *   row-unit head:     r[128] fp16 | c[128] fp16 | then the rows, each 16 b_i
  *                      bytes with the codes of columns 0..127 (b_i = 16 marks
  *                      an FP16 pivot row, 256 bytes), stored by decreasing
@@ -70,11 +71,12 @@ static double rne_div(double x, double d)
 {
     double n = rint(x / d);
     double e = x - n * d;
-    int odd = fmod(n, 2.0) != 0.0;
-    if (2.0 * e > d || (2.0 * e == d && odd))
-        n += 1.0;
-    else if (-2.0 * e > d || (-2.0 * e == d && odd))
-        n -= 1.0;
+    if (2.0 * e > d)
+        return n + 1.0;
+    if (-2.0 * e > d)
+        return n - 1.0;
+    if (2.0 * fabs(e) == d && fmod(n, 2.0) != 0.0)            /* a tie: the even neighbour */
+        return e > 0.0 ? n + 1.0 : n - 1.0;
     return n;
 }
 
@@ -93,24 +95,6 @@ size_t or_head_bytes(int unit_kind, const int8_t *rb)
     for (int i = 0; i < OR_D; i++)
         n += 16 * (size_t)rb[i];
     return n;
-}
-
-/* Byte offset of the stream holding element (i, j) and its bit position in it. */
-static size_t elem_stream(int unit_kind, const int8_t *rb, int i, int j, int *bitpos)
-{
-    int b = rb[i];
-    if (unit_kind == OR_UNIT_HEAD) {
-        size_t base = is_pivot_head(unit_kind, rb) ? 0 : 512;
-        size_t chunk = ((size_t)(j / 4) * 8 + (size_t)(i / 16)) * 4 + (size_t)(j % 4);
-        *bitpos = (i % 16) * b;
-        return base + chunk * 2 * (size_t)b;
-    }
-    size_t off = 512;                      /* rows of larger width, then earlier rows of width b */
-    for (int t = 0; t < OR_D; t++)
-        if (rb[t] > b || (rb[t] == b && t < i))
-            off += 16 * (size_t)rb[t];
-    *bitpos = j * b;
-    return off;
 }
 
 static void put_u16(uint8_t *p, uint16_t v) { p[0] = v & 0xFF; p[1] = v >> 8; }
@@ -138,12 +122,77 @@ static unsigned get_bits(const uint8_t *row, int pos, int b)
     return u;
 }
 
+/* Byte offset of the payload of row i of a row-unit segment: rows of larger
+ * width first, then earlier rows of width b_i (App. D fixes only the sizes). */
+static void row_offsets(const int8_t *rb, size_t *off)
+{
+    for (int i = 0; i < OR_D; i++) {
+        int b = rb[i];
+        off[i] = 512;
+        for (int r = 0; r < OR_D; r++)
+            if (rb[r] > b || (rb[r] == b && r < i))
+                off[i] += 16 * (size_t)rb[r];
+    }
+}
+
+/* Byte offset of bit t (0 <= t < b_i) of element (i, j) in a head segment, and
+ * that bit's position in the byte. row_off: row_offsets() for row units. */
+static size_t bit_addr(int unit_kind, const int8_t *rb, const size_t *row_off, int i, int j, int t,
+                       int *bit)
+{
+    int b = rb[i];
+    if (unit_kind == OR_UNIT_HEAD) {
+        /* The 16 codes of band g = i / 16 in column j form a chunk of 2b bytes,
+         * LSB-first. Column group w = j / 16 and lane l = 8 ((j / 4) % 4) + g own
+         * four chunks (columns 4 (j / 4) + 0..3), one stream of 2b 32-bit words;
+         * its 16-byte piece k sits at w * 256 b + k * 512 + 16 l. */
+        size_t base = is_pivot_head(unit_kind, rb) ? 0 : 512;
+        int w = j / 16, l = 8 * ((j / 4) % 4) + i / 16;
+        int L = (j % 4) * 16 * b + (i % 16) * b + t;              /* bit of the lane's stream */
+        int word = L / 32;
+        *bit = L % 8;
+        return base + (size_t)w * 256 * b + (size_t)(word / 4) * 512 + 16 * (size_t)l +
+               4 * (size_t)(word % 4) + (size_t)(L % 32) / 8;
+    }
+    *bit = (j * b + t) % 8;
+    return row_off[i] + (size_t)(j * b + t) / 8;
+}
+
+/* Element (i, j) of a head segment as a b_i-bit value: an offset-binary code,
+ * or the binary16 bits of an FP16 pivot (b_i = 16). */
+static void put_code(uint8_t *page, int unit_kind, const int8_t *rb, const size_t *row_off, int i,
+                     int j, unsigned u)
+{
+    for (int t = 0; t < rb[i]; t++) {
+        int bit;
+        uint8_t *p = page + bit_addr(unit_kind, rb, row_off, i, j, t, &bit);
+        if ((u >> t) & 1u)
+            *p |= (uint8_t)(1u << bit);
+        else
+            *p &= (uint8_t)~(1u << bit);
+    }
+}
+
+static unsigned get_code(const uint8_t *page, int unit_kind, const int8_t *rb, const size_t *row_off,
+                         int i, int j)
+{
+    unsigned u = 0;
+    for (int t = 0; t < rb[i]; t++) {
+        int bit;
+        const uint8_t *p = page + bit_addr(unit_kind, rb, row_off, i, j, t, &bit);
+        u |= (unsigned)((*p >> bit) & 1u) << t;
+    }
+    return u;
+}
+
 /* Unpack a head page into scales, integer codes and pivot values. For a
  * pivot head r and c are zero and every row is in `piv`. */
 void or_unpack_head(const uint8_t *page, int unit_kind, const int8_t *rb,
                     uint16_t *r, uint16_t *c, int8_t *codes, uint16_t *piv)
 {
     int ph = is_pivot_head(unit_kind, rb);
+    size_t off[OR_D];
+    row_offsets(rb, off);
     for (int i = 0; i < OR_D; i++) {
         r[i] = ph ? 0 : get_u16(page + 2 * i);
         c[i] = ph ? 0 : get_u16(page + 256 + 2 * i);
@@ -151,13 +200,11 @@ void or_unpack_head(const uint8_t *page, int unit_kind, const int8_t *rb,
     for (int i = 0; i < OR_D; i++) {
         int b = rb[i];
         for (int j = 0; j < OR_D; j++) {
-            int pos;
-            const uint8_t *stream = page + elem_stream(unit_kind, rb, i, j, &pos);
+            unsigned u = get_code(page, unit_kind, rb, off, i, j);
             if (b == OR_PIVOT_BITS) {
-                piv[i * OR_D + j] = get_u16(stream + pos / 8);
+                piv[i * OR_D + j] = (uint16_t)u;
                 codes[i * OR_D + j] = 0;
             } else {
-                unsigned u = get_bits(stream, pos, b);
                 codes[i * OR_D + j] = (int8_t)((int)u - (1 << (b - 1)));
                 piv[i * OR_D + j] = 0;
             }
@@ -267,13 +314,12 @@ void or_fit_debug(const float *X, int unit_kind, const int8_t *rb, const float *
 void or_encode_head(const float *X, int unit_kind, const int8_t *rb, const float *w,
                     int fit_iters, uint8_t *page)
 {
+    size_t off[OR_D];
+    row_offsets(rb, off);
     if (is_pivot_head(unit_kind, rb)) {             /* FP16 pivot head */
         for (int i = 0; i < OR_D; i++)
-            for (int j = 0; j < OR_D; j++) {
-                int pos;
-                uint8_t *stream = page + elem_stream(unit_kind, rb, i, j, &pos);
-                put_u16(stream + pos / 8, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
-            }
+            for (int j = 0; j < OR_D; j++)
+                put_code(page, unit_kind, rb, off, i, j, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
         return;
     }
     double r[OR_D], c[OR_D];
@@ -289,24 +335,23 @@ void or_encode_head(const float *X, int unit_kind, const int8_t *rb, const float
     for (int i = 0; i < OR_D; i++) {
         int b = rb[i];
         for (int j = 0; j < OR_D; j++) {
-            int pos;
-            uint8_t *stream = page + elem_stream(unit_kind, rb, i, j, &pos);
             if (b == OR_PIVOT_BITS) {
-                put_u16(stream + pos / 8, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
+                put_code(page, unit_kind, rb, off, i, j, or_fp16_encode(or_fp16_round(X[i * OR_D + j])));
                 continue;
             }
             double rz = r[i] * (double)zs_of(unit_kind, b);
             int qv = (int)level(X[i * OR_D + j], rz, c16[j], qmax_of(b));
-            put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1))));
+            put_code(page, unit_kind, rb, off, i, j, (unsigned)(qv + (1 << (b - 1))));
         }
     }
 }
 
 /* One persistent decode step of one head (App. C.3 steps 1-7): reconstruct,
- * X = D S + beta k (v^T - k^T D S), y = X^T q, refit, requantize in place. */
+ * X = D S + beta k (v^T - k^T D S), y = X^T q, refit, requantize in place.
+ * delta (optional, [128]): the residual v_j - u_j of the retrieval. */
 void or_step_head(uint8_t *page, int unit_kind, const int8_t *rb, const float *w,
                   int fit_iters, const float *q, const float *k, const float *v,
-                  float beta, const float *gate, int gate_per_row, float *y)
+                  float beta, const float *gate, int gate_per_row, float *y, double *delta)
 {
     double *S = malloc(sizeof(double) * OR_N);
     float *X = malloc(sizeof(float) * OR_N);
@@ -333,6 +378,9 @@ void or_step_head(uint8_t *page, int unit_kind, const int8_t *rb, const float *w
             acc += (double)q[i] * (double)X[i * OR_D + j];
         y[j] = (float)acc;
     }
+    if (delta)                                                 /* v - k^T D S_hat, optional */
+        for (int j = 0; j < OR_D; j++)
+            delta[j] = (double)v[j] - u[j];
     or_encode_head(X, unit_kind, rb, w, fit_iters, page);
     free(S);
     free(X);

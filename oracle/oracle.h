@@ -70,7 +70,7 @@ void or_decode_head(const uint8_t *page, int unit_kind, const int8_t *row_bits, 
 void or_decode_head_f32(const uint8_t *page, int unit_kind, const int8_t *row_bits, float *S);
 void or_step_head(uint8_t *page, int unit_kind, const int8_t *row_bits, const float *w,
                   int fit_iters, const float *q, const float *k, const float *v,
-                  float beta, const float *gate, int gate_per_row, float *y);
+                  float beta, const float *gate, int gate_per_row, float *y, double *delta);
 void or_fit_debug(const float *X, int unit_kind, const int8_t *row_bits, const float *w,
                   int fit_iters, double *r, double *c_iter, int8_t *z_last);
 void or_unpack_head(const uint8_t *page, int unit_kind, const int8_t *row_bits,
@@ -113,7 +113,8 @@ void or_pool_step(int unit_kind, int Hk, int Hv, int gate_per_row, const int8_t 
                   const float *layer_w, int fit_iters, const uint64_t *layer_head_off,
                   uint64_t slot_stride, uint8_t *pool, const int32_t *slots, int B,
                   const float *q, const float *k, const float *v, const float *beta,
-                  const float *gate, float *y);
+                  const float *gate, float *y,
+                  double *delta);
 void or_pool_step_units(int unit_kind, int Hk, int Hv, int gate_per_row,
                         const int8_t *layer_row_bits, const float *layer_w, int fit_iters,
                         const uint64_t *layer_head_off, uint64_t slot_stride, uint8_t *pool,

@@ -10,10 +10,12 @@
 // group, whose result lane rg holds for column rg >> 1 of its group. Only the
 // row reduction of the row factors crosses warps, through shared memory.
 //
-// Page chunks: the 16 codes of band g in column j take 2b bytes; chunk index
-// ((j / 4) * 8 + g) * 4 + j % 4, so thread tid's four chunks are the 8b
-// contiguous bytes of block tid and the 32 lanes of a warp read 32 consecutive
-// blocks (no shared-memory bank conflicts beyond the minimum wavefronts).
+// Page codes: the 16 codes of band g in column j form a chunk of 2b bytes; a
+// thread's four chunks (columns 16w + 4cg + 0..3 of band rg) are one stream of
+// 2b words, stored as B/2 16-byte pieces interleaved over the warp's 32 lanes:
+// piece k of lane l of warp w at w * 256 B + k * 512 + 16 l. Every 16-byte
+// load or store of a warp then covers 512 contiguous bytes, with no bank
+// conflicts for any width.
 // Per-row constants sit in shared memory with a pad of 4 floats after every
 // band of 16 rows, so the 8 bands a warp reads hit distinct banks.
 //
@@ -39,8 +41,8 @@ constexpr int kPad = 160;                              // padded per-row array: 
 
 // ------------------------------------------------------------ shared layout
 constexpr int kOffBars = 0;                            // uint64 [8]
-constexpr int kOffRed = 128;                           // float [8][128] row partial sums per warp
-constexpr int kOffRows = kOffRed + 8 * 128 * 4;        // float [6][kPad] per-row constants
+constexpr int kOffRed = 128;                           // float [8][kPad] row partial sums per warp
+constexpr int kOffRows = kOffRed + 8 * kPad * 4;       // float [6][kPad] per-row constants
 constexpr int kMaxHv = 256;                            // value heads per layer (launch check)
 constexpr int kOffHead = kOffRows + 6 * kPad * 4;      // u64 off | u32 bytes | u8 bits | u8 key head
 constexpr int kOffStages = (kOffHead + kMaxHv * 14 + 127) / 128 * 128;
@@ -158,16 +160,16 @@ __device__ __forceinline__ void row_sum_scatter(const float (&v)[16], int cg, fl
         out[t] = (b1 ? a8[4 + t] : a8[t]) + __shfl_xor_sync(0xffffffffu, b1 ? a8[t] : a8[4 + t], 16);
 }
 
-// ---- page blocks: thread tid's four chunks, 8B contiguous bytes ----
+// ---- page streams: a thread's four chunks as B/2 interleaved 16-byte pieces ----
 template <int B>
-__device__ __forceinline__ uint8_t *block_ptr(uint8_t *page, int tid) {
-    return page + (B == kPivot ? 0 : 512) + tid * 8 * B;
+__device__ __forceinline__ uint8_t *stream_base(uint8_t *page, const T &t) {
+    return page + (B == kPivot ? 0 : 512) + t.w * 256 * B + 16 * t.l;
 }
 template <int B>
 __device__ __forceinline__ void load_block(const uint8_t *p, uint32_t (&wd)[2 * B]) {
 #pragma unroll
     for (int k = 0; k < B / 2; k++) {
-        const uint4 a = ((const uint4 *)p)[k];
+        const uint4 a = *(const uint4 *)(p + 512 * k);
         wd[4 * k] = a.x; wd[4 * k + 1] = a.y; wd[4 * k + 2] = a.z; wd[4 * k + 3] = a.w;
     }
 }
@@ -175,7 +177,7 @@ template <int B>
 __device__ __forceinline__ void store_block(uint8_t *p, const uint32_t (&wd)[2 * B]) {
 #pragma unroll
     for (int k = 0; k < B / 2; k++)
-        ((uint4 *)p)[k] = make_uint4(wd[4 * k], wd[4 * k + 1], wd[4 * k + 2], wd[4 * k + 3]);
+        *(uint4 *)(p + 512 * k) = make_uint4(wd[4 * k], wd[4 * k + 1], wd[4 * k + 2], wd[4 * k + 3]);
 }
 
 // Scale of the high code of a pair as placed by code_pair (2^B, or 1 for B = 8).
@@ -304,7 +306,7 @@ __device__ __forceinline__ void final_codes(const T &t, uint8_t *page, const uin
         }
         pack_codes<B>(f, wd, c);
     }
-    store_block<B>(block_ptr<B>(page, t.tid), wd);
+    store_block<B>(stream_base<B>(page, t), wd);
 }
 
 // ---------------------------------------------------------------- the fit
@@ -331,7 +333,7 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
     {
         float part[4];
         row_sum_scatter(rs, t.cg, part);
-        *(float4 *)&S.red[t.w * 128 + t.row(8 * (t.cg & 1) + 4 * (t.cg >> 1))] =
+        *(float4 *)&S.red[t.w * kPad + prow(t.row(8 * (t.cg & 1) + 4 * (t.cg >> 1)))] =
             make_float4(part[0], part[1], part[2], part[3]);
     }
     __syncthreads();
@@ -340,7 +342,7 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         const int i = t.tid;
         float sz = 0.f;
 #pragma unroll
-        for (int wv = 0; wv < 8; wv++) sz += S.red[wv * 128 + i];
+        for (int wv = 0; wv < 8; wv++) sz += S.red[wv * kPad + prow(i)];
         const float a = scaled ? S.rA[prow(i)] : 1.f;
         const float m = (a * sz) * (1.0f / 128.0f);
         const float rf = __half2float(__float2half_rn(
@@ -416,7 +418,7 @@ __device__ __forceinline__ void pack_pivot(const T &t, uint8_t *page, const uint
         for (int m = 0; m < 8; m++)
             wd[8 * c + m] = (uint32_t)f16_bits(f16_round_sat(a * f2lo(x2[m][c]))) |
                             ((uint32_t)f16_bits(f16_round_sat(a * f2hi(x2[m][c]))) << 16);
-    store_block<kPivot>(block_ptr<kPivot>(page, t.tid), wd);
+    store_block<kPivot>(stream_base<kPivot>(page, t), wd);
 }
 
 // Reconstruct the column-scaled codes c_j q_ij (exact in fp32) or the FP16
@@ -424,7 +426,7 @@ __device__ __forceinline__ void pack_pivot(const T &t, uint8_t *page, const uint
 template <int B>
 __device__ __forceinline__ void load_tile(const T &t, const uint8_t *page, uint64_t (&x2)[8][4]) {
     uint32_t wd[2 * B];
-    load_block<B>(block_ptr<B>((uint8_t *)page, t.tid), wd);
+    load_block<B>(stream_base<B>((uint8_t *)page, t), wd);
     if constexpr (B == kPivot) {
 #pragma unroll
         for (int c = 0; c < 4; c++)

@@ -43,6 +43,14 @@ def _widths(rng, unit, b=None):
     return rb
 
 
+def _head_streams(codes, b):
+    """The 256 per-lane streams (8b bytes each) of a head's code region, ordered
+    [column group w][lane l = 8 cg + g]: piece k (16 bytes) of lane l of group w
+    sits at w * 256 b + k * 512 + 16 l."""
+    return (np.asarray(codes).reshape(8, b // 2, 32, 16).transpose(0, 2, 1, 3)
+            .reshape(8, 32, 8 * b))
+
+
 def _check_nearest_levels(oracle, X, unit, rb, page):
     r16, c16, codes, piv = oracle.unpack_head(page, unit, rb)
     r, c = _f16(r16), _f16(c16)
@@ -86,8 +94,8 @@ def test_pivot_head_is_fp16(oracle, rng):
     rb = np.full(D, PIV, np.int8)
     page = oracle.encode_head(X, HEAD, rb, _w(rng))
     assert page.size == D * D * 2
-    # chunks [column group t][band g][column 4t + c][row 16g + r]
-    vals = page.view(np.float16).reshape(32, 8, 4, 16).transpose(1, 3, 0, 2).reshape(D, D)
+    vals = _head_streams(page, 16).view(np.float16).reshape(8, 4, 8, 4, 16)   # [w][cg][g][c][r]
+    vals = vals.transpose(2, 4, 0, 1, 3).reshape(D, D)
     ref = np.float16(np.clip(X, -65504, 65504))
     assert np.array_equal(vals.astype(np.float64), ref.astype(np.float64))
 
@@ -95,8 +103,9 @@ def test_pivot_head_is_fp16(oracle, rng):
 @pytest.mark.parametrize("b", [2, 4, 6, 8])
 def test_bit_layout_with_independent_unpacker(oracle, rng, b):
     """Head units: offset-binary codes u = q + 2^(b-1), LSB-first, in chunks of
-    the 16 codes of one band of rows (16g..16g+15) in one column, ordered by
-    column group (4 columns), band, column within the group."""
+    the 16 codes of one band of rows (16g..16g+15) in one column; the four chunks
+    of a band in 4 adjacent columns form one stream, stored as 16-byte pieces
+    interleaved over the 32 streams of each group of 16 columns."""
     X = _state(rng)
     rb = np.full(D, b, np.int8)
     page = oracle.encode_head(X, HEAD, rb, _w(rng))
@@ -104,9 +113,9 @@ def test_bit_layout_with_independent_unpacker(oracle, rng, b):
     r16, c16, codes, _ = oracle.unpack_head(page, HEAD, rb)
     assert np.array_equal(page[:256].view(np.uint16), r16)
     assert np.array_equal(page[256:512].view(np.uint16), c16)
-    bits = np.unpackbits(page[512:].reshape(8 * D, 2 * b), axis=1, bitorder="little")
-    u = (bits.reshape(32, 8, 4, 16, b) * (1 << np.arange(b))).sum(-1)   # [group][band][c][row in band]
-    u = u.transpose(1, 3, 0, 2).reshape(D, D)
+    bits = np.unpackbits(_head_streams(page[512:], b), axis=-1, bitorder="little")
+    u = (bits.reshape(8, 4, 8, 4, 16, b) * (1 << np.arange(b))).sum(-1)   # [w][cg][g][c][r]
+    u = u.transpose(2, 4, 0, 1, 3).reshape(D, D)
     assert np.array_equal(u - 2 ** (b - 1), codes.astype(np.int64))
     assert u.min() >= 1
 

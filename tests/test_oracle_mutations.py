@@ -65,13 +65,13 @@ MUTANTS = [
      "                double a = fabs((double)X[i * OR_D + j]) / rz[i];"),
     ("codes_floored", "codec.c", "    return clampd(rne_div((double)x, r_zs * c), -qm, qm);",
      "    return clampd(floor((double)x / (r_zs * c)), -qm, qm);"),
-    ("code_ties_up", "codec.c", "    if (2.0 * e > d || (2.0 * e == d && odd))",
-     "    if (2.0 * e > d || 2.0 * e == d)"),
+    ("code_ties_to_odd", "codec.c", "    if (2.0 * fabs(e) == d && fmod(n, 2.0) != 0.0)",
+     "    if (2.0 * fabs(e) == d && fmod(n, 2.0) == 0.0)"),
     ("code_clip_qmax_plus_one", "codec.c", "    return clampd(rne_div((double)x, r_zs * c), -qm, qm);",
      "    return clampd(rne_div((double)x, r_zs * c), -qm - 1, qm + 1);"),
     ("offset_binary_bias", "codec.c",
-     "            put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1))));",
-     "            put_bits(stream, pos, b, (unsigned)(qv + (1 << (b - 1)) - 1));"),
+     "            put_code(page, unit_kind, rb, off, i, j, (unsigned)(qv + (1 << (b - 1))));",
+     "            put_code(page, unit_kind, rb, off, i, j, (unsigned)(qv + (1 << (b - 1)) - 1));"),
     ("final_codes_unrounded_c", "codec.c",
      "            int qv = (int)level(X[i * OR_D + j], rz, c16[j], qmax_of(b));",
      "            int qv = (int)level(X[i * OR_D + j], rz, c[j], qmax_of(b));"),
@@ -129,10 +129,14 @@ MUTANTS = [
     ("pivot_rows_in_fit", "codec.c", "        in_fit[i] = (b != OR_PIVOT_BITS);", "        in_fit[i] = 1;"),
     ("bits_msb_first", "codec.c", "        if ((u >> t) & 1u)\n            row[p >> 3] |=",
      "        if ((u >> (b - 1 - t)) & 1u)\n            row[p >> 3] |="),
-    ("rows_stored_ascending", "codec.c", "        if (rb[t] > b || (rb[t] == b && t < i))",
-     "        if (rb[t] < b || (rb[t] == b && t < i))"),
-    ("band_of_row", "codec.c", "        size_t chunk = ((size_t)(j / 4) * 8 + (size_t)(i / 16)) * 4 + (size_t)(j % 4);",
-     "        size_t chunk = ((size_t)(j / 4) * 8 + (size_t)(i % 8)) * 4 + (size_t)(j % 4);"),
+    ("rows_stored_ascending", "codec.c", "            if (rb[r] > b || (rb[r] == b && r < i))",
+     "            if (rb[r] < b || (rb[r] == b && r < i))"),
+    ("band_of_row", "codec.c", "        int w = j / 16, l = 8 * ((j / 4) % 4) + i / 16;",
+     "        int w = j / 16, l = 8 * ((j / 4) % 4) + i % 8;"),
+    ("pieces_contiguous_per_lane", "codec.c", "(size_t)(word / 4) * 512 + 16 * (size_t)l +",
+     "(size_t)(word / 4) * 16 + 16 * (size_t)l +"),
+    ("code_bits_msb_first", "codec.c", "        if ((u >> t) & 1u)\n            *p |= (uint8_t)(1u << bit);",
+     "        if ((u >> (rb[i] - 1 - t)) & 1u)\n            *p |= (uint8_t)(1u << bit);"),
     ("fp16_subnormal_scale", "numerics.c", "        return s | (uint16_t)(a / ldexp(1.0, -24));   /* subnormal: fraction counts 2^-24 */",
      "        return s | (uint16_t)(a / ldexp(1.0, -23));   /* subnormal: fraction counts 2^-24 */"),
     ("row_pivot_risk_without_fp16", "plan.c",
