@@ -309,6 +309,22 @@ __device__ __forceinline__ void final_codes(const T &t, uint8_t *page, const uin
     store_block<B>(stream_base<B>(page, t), wd);
 }
 
+// Approximate reciprocal and square root (the SFU's, within about 1 ulp) where
+// the result only shapes a scale: the row factor's square root (rounded to FP16
+// next), rho_i and the column scale of the first fixed-code pass. The reciprocal
+// of the stored FP16 column scale, which takes the final code decisions, stays
+// correctly rounded.
+__device__ __forceinline__ float rcp_approx(float x) {
+    float d;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(d) : "f"(x));
+    return d;
+}
+__device__ __forceinline__ float sqrt_approx(float x) {
+    float d;
+    asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(d) : "f"(x));
+    return d;
+}
+
 // ---------------------------------------------------------------- the fit
 // Key-Row-Aware Dual-axis Fitting of the register tile (Sec. 4.3, App. C.1)
 // and packing into the page (App. C.3 step 6). The tile holds Z with
@@ -346,8 +362,8 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         const float a = scaled ? S.rA[prow(i)] : 1.f;
         const float m = (a * sz) * (1.0f / 128.0f);
         const float rf = __half2float(__float2half_rn(
-            fminf(fmaxf(__fmul_rn(sqrtf(m), wisv[i]), kF16Min), kF16Max)));
-        S.rRho[prow(i)] = __frcp_rn(rf) * a;              // X' = rho_i X = (rho_i a_i) Z
+            fminf(fmaxf(__fmul_rn(sqrt_approx(m), wisv[i]), kF16Min), kF16Max)));
+        S.rRho[prow(i)] = rcp_approx(rf) * a;             // X' = rho_i X = (rho_i a_i) Z
         S.rAl[prow(i)] = w2v[i] * (rf * rf);              // w_i^2 r_i^2
         page_r[i] = f16_bits(rf);
     }
@@ -369,10 +385,10 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
     }
     // this lane's column (own_col): its max, its current scale, its reciprocal
     const float mx = col_max_scatter(cm, t.rg);
-    const float c0 = __fmul_rn(mx, __frcp_rn(fqm));
+    const float c0 = __fmul_rn(mx, 1.0f / fqm);
     const bool clip0 = __any_sync(0xffffffffu, c0 > kF16Max);   // start capped: codes may clip
     float cc = fminf(fmaxf(c0, kF16Min), kF16Max);
-    float gi = __frcp_rn(cc);
+    float gi = rcp_approx(cc);
     uint64_t g[4];
 #pragma unroll
     for (int c = 0; c < 4; c++) g[c] = f2s(col_gather(gi, t, c));
@@ -391,7 +407,7 @@ __device__ __forceinline__ void fit_pack(const T &t, const Smem &S, uint8_t *pag
         // num and den carry fp32 summation error already; a 2-ulp quotient adds nothing
         if (den > 0.f) cc = fminf(fmaxf(__fdividef(num, den), kF16Min), kF16Max);
         if (it + 1 < fit_iters) {
-            gi = __frcp_rn(cc);
+            gi = rcp_approx(cc);
         } else {
             // storage precision of c; codes can clip only where max |X'| / c >= qmax + 1/2
             const float cf = __half2float(__float2half_rn(cc));
