@@ -211,3 +211,46 @@ def test_pool_step_is_the_per_unit_step(oracle, rng):
     for s in set(range(n_slots)) - set(slots.tolist()):
         seg = slice(s * plan.slot_stride, (s + 1) * plan.slot_stride)
         assert np.array_equal(pool[seg], before[seg])
+
+
+@pytest.mark.parametrize("gate_kind", ["scalar", "channel"])
+def test_reported_residual_matches_the_readout(oracle, rng, gate_kind):
+    """The residual delta = v - k^T D S_hat that the step reports (App. C.3 step 2)
+    is the one its update applied: with X = D S_hat + beta k delta^T, the readout
+    satisfies y - (D S_hat)^T q = beta (q . k) delta (Eq. compressed_recurrence),
+    up to the fp32 rounding of X."""
+    Hk, Hv, n_slots = 2, 4, 3
+    slots = np.array([2, 0], np.int32)
+    B = len(slots)
+    unit = HEAD if gate_kind == "scalar" else ROW
+    cands = (4, 6, 8)
+    units = Hv if unit == HEAD else Hv * D
+    dist = np.sort(np.exp(rng.normal(0, 1, (units, 4))), axis=1)[:, ::-1].copy()
+    plan = oracle.make_plan(unit, 1, Hk, Hv, 6, cands, 0, 64, 1,
+                            np.exp(rng.normal(0, 1, (1, Hv, D))).astype(np.float32),
+                            rng.normal(-0.02, 0.01, units), dist)
+    pool = np.zeros(n_slots * plan.slot_stride, np.uint8)
+    oracle.pool_encode(plan, pool, 0, slots, rng.standard_normal((B, Hv, D, D)).astype(np.float32))
+    S_hat = oracle.pool_decode(plan, pool, 0, slots).astype(np.float64)
+
+    class Inp:
+        pass
+    inp = Inp()
+    inp.q = rng.standard_normal((B, Hk, D)).astype(np.float32)
+    inp.k = rng.standard_normal((B, Hk, D)).astype(np.float32)
+    inp.k /= np.linalg.norm(inp.k, axis=-1, keepdims=True)
+    inp.v = rng.standard_normal((B, Hv, D)).astype(np.float32)
+    inp.beta = rng.uniform(0.1, 0.9, (B, Hv)).astype(np.float32)
+    gshape = (B, Hv) if unit == HEAD else (B, Hv, D)
+    inp.gate = rng.uniform(0.9, 0.999, gshape).astype(np.float32)
+    y, delta = oracle.pool_step(plan, pool, 0, slots, inp, with_delta=True)
+    q = np.repeat(inp.q.astype(np.float64), Hv // Hk, axis=1)
+    k = np.repeat(inp.k.astype(np.float64), Hv // Hk, axis=1)
+    g = inp.gate.astype(np.float64)
+    g = g[..., None, None] if unit == HEAD else g[..., :, None]
+    base = np.einsum("bhi,bhij->bhj", q, g * S_hat)
+    lhs = y.astype(np.float64) - base
+    rhs = inp.beta.astype(np.float64)[..., None] * np.einsum("bhi,bhi->bh", q, k)[..., None] * delta
+    scale = np.einsum("bhi,bhij->bhj", np.abs(q), np.abs(g * S_hat)).max(axis=-1, keepdims=True)
+    assert np.all(np.abs(lhs - rhs) <= 1e-5 * scale)
+    assert np.abs(rhs).max() > 1e-3 * np.abs(lhs).max()       # the term is not negligible
