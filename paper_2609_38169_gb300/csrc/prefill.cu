@@ -57,7 +57,7 @@ constexpr uint32_t kIdescP3 = tc::idesc_tf32(128, 32);
 // row groups kSbo128 / kSbo32 apart for K = 128 / 32.
 constexpr int kLbo = 144;
 constexpr int kSbo128 = 32 * kLbo;                     // 4608
-constexpr int kSbo32 = 8 * kLbo;                       // 1152
+constexpr int kSbo32 = 8 * kLbo + 16;                  // 1168: 16-byte rows of 8 row groups in distinct banks
 // P0 reads 128 rows of A from B1: rows 64..127 fall on B1l and B3 (valid
 // memory; their results are unused).
 constexpr int kOffB1h = 0;                             // [K~ ; Q~] head: 64 rows x K 128
@@ -70,7 +70,7 @@ constexpr int kOffB4h = kOffB2l + 16 * kSbo32;         // Bm head: 32 rows (t) x
 constexpr int kOffB4l = kOffB4h + 4 * kSbo32;
 constexpr int kOffV = kOffB4l + 4 * kSbo32;            // float [C][128] V
 constexpr int kOffG = kOffV + C * 128 * 4;             // float [C][128] cumulative gates
-constexpr int kOffA = kOffG + C * 128 * 4;             // float [C][C] A (strict lower)
+constexpr int kOffA = kOffG + C * 128 * 4;             // float [C][C] A^T: row s holds A_ts over t (t > s)
 constexpr int kOffBeta = kOffA + C * C * 4;            // float [C]
 constexpr int kOffBar = kOffBeta + C * 4;              // uint64 mbarrier
 constexpr int kOffTmem = kOffBar + 8;                  // u32 tensor-memory base
@@ -87,6 +87,19 @@ __device__ __forceinline__ void put_split(uint8_t *hi_base, uint8_t *lo_base, in
     tc::split_tf32(x, hi, lo);
     *(float *)(hi_base + off) = hi;
     *(float *)(lo_base + off) = lo;
+}
+// Four consecutive K elements of one row (off 16-byte aligned).
+__device__ __forceinline__ void put_split4(uint8_t *hi_base, uint8_t *lo_base, int off, float4 x) {
+    float4 hi, lo;
+    tc::split_tf32(x.x, hi.x, lo.x);
+    tc::split_tf32(x.y, hi.y, lo.y);
+    tc::split_tf32(x.z, hi.z, lo.z);
+    tc::split_tf32(x.w, hi.w, lo.w);
+    *(float4 *)(hi_base + off) = hi;
+    *(float4 *)(lo_base + off) = lo;
+}
+__device__ __forceinline__ float4 mul4(float4 a, float4 b) {
+    return make_float4(a.x * b.x, a.y * b.y, a.z * b.z, a.w * b.w);
 }
 
 struct Args {
@@ -133,23 +146,24 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
     };
     // This thread's share of a chunk's operands, loaded one chunk ahead (their
     // global-memory latency overlaps the previous chunk's tensor-core work):
-    // key channel ci at tokens tb, tb + 2, ..., tb + 30 of k, q, v; threads
-    // 0..127 the chunk's gates of channel ci, threads 128..159 one beta each.
-    // Missing tokens of a ragged tail are the identity step (gate 1, beta 0,
-    // zero k, q, v).
-    const int ci = tid & 127, tb = tid >> 7;
-    float kv[C / 2], qv[C / 2], vv[C / 2], dg[C], bt = 0.f;
+    // key channels 4 cq .. 4 cq + 3 at tokens 4 tq .. 4 tq + 3 of k, q, v (one
+    // 16-byte load each); threads 0..127 the chunk's gates of channel ci,
+    // threads 128..159 one beta each. Missing tokens of a ragged tail are the
+    // identity step (gate 1, beta 0, zero k, q, v).
+    const int ci = tid & 127, cq = tid & 31, tq = tid >> 5;
+    float4 kv[4], qv[4], vv[4];
+    float dg[C], bt = 0.f;
     const auto fetch = [&](int it, int c0) {
         const int fb = it / a.Hv, fh = it - fb * a.Hv, fhk = fh / grp, fn = min(C, a.T - c0);
 #pragma unroll
-        for (int u = 0; u < C / 2; u++) {
-            const int t = tb + 2 * u;
-            kv[u] = qv[u] = vv[u] = 0.f;
+        for (int m = 0; m < 4; m++) {
+            const int t = 4 * tq + m;
+            kv[m] = qv[m] = vv[m] = make_float4(0.f, 0.f, 0.f, 0.f);
             if (t < fn) {
                 const size_t tok = (size_t)fb * a.T + c0 + t;
-                kv[u] = a.k[(tok * a.Hk + fhk) * 128 + ci];
-                qv[u] = a.q[(tok * a.Hk + fhk) * 128 + ci];
-                vv[u] = a.v[(tok * a.Hv + fh) * 128 + ci];
+                kv[m] = *(const float4 *)&a.k[(tok * a.Hk + fhk) * 128 + 4 * cq];
+                qv[m] = *(const float4 *)&a.q[(tok * a.Hk + fhk) * 128 + 4 * cq];
+                vv[m] = *(const float4 *)&a.v[(tok * a.Hv + fh) * 128 + 4 * cq];
             }
         }
         if (tid < 128) {
@@ -199,20 +213,31 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
                 bet[tid - 128] = bt;
             }
             __syncthreads();
-            // Element-wise: V, and the split operands [K~ ; Q~], K^ and K_bar^T.
+            // Element-wise: V, and the split operands [K~ ; Q~], K^ and K_bar^T,
+            // four consecutive K elements per store.
             {
-                const int i = ci;
-                const float gC = G[(C - 1) * 128 + i];
+                const int c4 = 4 * cq;
+                const float4 gC = *(const float4 *)&G[(C - 1) * 128 + c4];
+                float kb[4][4];                               // K_bar^T: [channel][token]
 #pragma unroll
-                for (int u = 0; u < C / 2; u++) {
-                    const int t = tb + 2 * u;
-                    const float g = G[t * 128 + i], rg = __fdividef(1.0f, g);   // within 2 ulp
-                    V[t * 128 + i] = vv[u];
-                    put_split(B1h, B1l, core_off(t, i, kSbo128), g * kv[u]);        // K~
-                    put_split(B1h, B1l, core_off(C + t, i, kSbo128), g * qv[u]);    // Q~
-                    put_split(B3h, B3l, core_off(t, i, kSbo128), kv[u] * rg);       // K^
-                    put_split(B2h, B2l, core_off(i, t, kSbo32), kv[u] * (gC * rg)); // K_bar^T
+                for (int m = 0; m < 4; m++) {
+                    const int t = 4 * tq + m;
+                    const float4 g = *(const float4 *)&G[t * 128 + c4];
+                    const float4 rg = make_float4(__fdividef(1.0f, g.x), __fdividef(1.0f, g.y),   // within 2 ulp
+                                                  __fdividef(1.0f, g.z), __fdividef(1.0f, g.w));
+                    *(float4 *)&V[t * 128 + c4] = vv[m];
+                    put_split4(B1h, B1l, core_off(t, c4, kSbo128), mul4(g, kv[m]));        // K~
+                    put_split4(B1h, B1l, core_off(C + t, c4, kSbo128), mul4(g, qv[m]));    // Q~
+                    put_split4(B3h, B3l, core_off(t, c4, kSbo128), mul4(kv[m], rg));       // K^
+                    kb[0][m] = kv[m].x * (gC.x * rg.x);
+                    kb[1][m] = kv[m].y * (gC.y * rg.y);
+                    kb[2][m] = kv[m].z * (gC.z * rg.z);
+                    kb[3][m] = kv[m].w * (gC.w * rg.w);
                 }
+#pragma unroll
+                for (int e = 0; e < 4; e++)
+                    put_split4(B2h, B2l, core_off(c4 + e, 4 * tq, kSbo32),
+                               make_float4(kb[e][0], kb[e][1], kb[e][2], kb[e][3]));
             }
             fence_async_smem();                           // operands visible to the tensor cores
             __syncthreads();
@@ -238,15 +263,17 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
                 alive = false;
                 break;
             }
-            // A = strict lower of diag(beta) K~ K^T (row t = lane t) and Bm =
-            // lower (with diagonal) of Q~ K^T (row t = lane 32 + t), Bm split as an operand.
+            // A = strict lower of diag(beta) K~ K^T (row t = lane t), stored
+            // transposed (a warp's store is one row of A^T: no bank conflicts), and
+            // Bm = lower (with diagonal) of Q~ K^T (row t = lane 32 + t), Bm split
+            // as an operand.
             if (w < 2) {
                 float d[32];
                 tc::ld32(tl + kColP0, d);
                 if (w == 0) {
                     const float bt = bet[l];
 #pragma unroll
-                    for (int s = 0; s < C; s++) A[l * C + s] = s < l ? bt * d[s] : 0.f;
+                    for (int s = 0; s < C; s++) A[s * C + l] = s < l ? bt * d[s] : 0.f;
                 } else {
 #pragma unroll
                     for (int s = 0; s < C; s++) put_split(B4h, B4l, core_off(l, s, kSbo32), s <= l ? d[s] : 0.f);
@@ -255,21 +282,25 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
             }
             __syncthreads();                              // A visible; P0's columns free for W
             if (half == 0) {
-                // W = (I + A)^-1 diag(beta) (V - K~ S_0), value column j.
-                float x[32], wv[32];
-                tc::ld32(tl + kColX, x);
+                // W = (I + A)^-1 diag(beta) (V - K~ S_0), value column j, by forward
+                // substitution in column order: once w_s is final it is taken out
+                // of every later row (independent updates, so the dependent chain
+                // is one fma per token).
+                float wv[32];
+                tc::ld32(tl + kColX, wv);
 #pragma unroll
-                for (int t = 0; t < C; t++) {
-                    float acc = bet[t] * (V[t * 128 + j] - x[t]);
+                for (int t = 0; t < C; t++) wv[t] = bet[t] * (V[t * 128 + j] - wv[t]);
 #pragma unroll
-                    for (int s4 = 0; 4 * s4 < t; s4++) {           // A row t, four at a time
-                        const float4 a4 = ((const float4 *)(A + t * C))[s4];
+                for (int s = 0; s < C - 1; s++) {
+                    const float ws = wv[s];
+#pragma unroll
+                    for (int t4 = (s + 1) / 4; t4 < C / 4; t4++) {    // row s of A^T, four at a time
+                        const float4 a4 = ((const float4 *)(A + s * C))[t4];
                         const float av[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
                         for (int e = 0; e < 4; e++)
-                            if (4 * s4 + e < t) acc -= av[e] * wv[4 * s4 + e];
+                            if (4 * t4 + e > s) wv[4 * t4 + e] = fmaf(-av[e], ws, wv[4 * t4 + e]);
                     }
-                    wv[t] = acc;
                 }
                 float hi[32], lo[32];
 #pragma unroll
