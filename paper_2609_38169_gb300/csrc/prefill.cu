@@ -32,7 +32,8 @@
 //   [384, 416) (K~ S_0)^T | [416, 448) (Q~ S_0)^T, then Y^T |
 //   [448, 480) P0 result, then W^T head | [480, 512) W^T rest.
 // Warps w and w + 4 share tensor-memory lanes 32 (w % 4) ..: the first four
-// warps solve for W while the last four scale the state by g_C.
+// warps solve for W while the last four scale the state by g_C. While P2 and
+// P3 run, all warps prepare the next chunk's operands.
 #include "async.cuh"
 #include "device.cuh"
 #include "internal.h"
@@ -179,7 +180,65 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
             bt = t < fn ? a.beta[((size_t)fb * a.T + c0 + t) * a.Hv + fh] : 0.f;
         }
     };
-    if ((int)blockIdx.x < a.items) fetch(blockIdx.x, 0);
+    // One chunk's cumulative gates g_t per key channel (multiplied in token
+    // order), beta, V and the split operands [K~ ; Q~] and K^, from the fetched
+    // registers, four consecutive K elements per store. K_bar^T, P2's operand,
+    // stays in kb until put_kbar (the previous chunk's P2 may still read it).
+    float kb[4][4];                                        // K_bar^T: [channel][token]
+    const auto prep = [&]() {
+        if (tid < 128) {
+            float g = 1.f;
+#pragma unroll
+            for (int t = 0; t < C; t++) {
+                g = fmaxf(g * dg[t], 1e-30f);             // keeps K / g finite
+                G[t * 128 + tid] = g;
+            }
+        } else if (tid < 128 + C) {
+            bet[tid - 128] = bt;
+        }
+        __syncthreads();
+        const int c4 = 4 * cq;
+        const float4 gC = *(const float4 *)&G[(C - 1) * 128 + c4];
+#pragma unroll
+        for (int m = 0; m < 4; m++) {
+            const int t = 4 * tq + m;
+            const float4 g = *(const float4 *)&G[t * 128 + c4];
+            const float4 rg = make_float4(__fdividef(1.0f, g.x), __fdividef(1.0f, g.y),   // within 2 ulp
+                                          __fdividef(1.0f, g.z), __fdividef(1.0f, g.w));
+            *(float4 *)&V[t * 128 + c4] = vv[m];
+            put_split4(B1h, B1l, core_off(t, c4, kSbo128), mul4(g, kv[m]));        // K~
+            put_split4(B1h, B1l, core_off(C + t, c4, kSbo128), mul4(g, qv[m]));    // Q~
+            put_split4(B3h, B3l, core_off(t, c4, kSbo128), mul4(kv[m], rg));       // K^
+            kb[0][m] = kv[m].x * (gC.x * rg.x);
+            kb[1][m] = kv[m].y * (gC.y * rg.y);
+            kb[2][m] = kv[m].z * (gC.z * rg.z);
+            kb[3][m] = kv[m].w * (gC.w * rg.w);
+        }
+    };
+    const auto put_kbar = [&]() {
+#pragma unroll
+        for (int e = 0; e < 4; e++)
+            put_split4(B2h, B2l, core_off(4 * cq + e, 4 * tq, kSbo32),
+                       make_float4(kb[e][0], kb[e][1], kb[e][2], kb[e][3]));
+    };
+    // This CTA's chunks in order: (item, first token); fi, fc is the chunk
+    // whose inputs the registers hold.
+    int fi = blockIdx.x, fc = 0;
+    const auto advance = [&]() {
+        fc += C;
+        if (fc >= a.T) {
+            fi += gridDim.x;
+            fc = 0;
+        }
+    };
+    // Prologue: the first chunk prepared, the second fetched.
+    if (fi < a.items) {
+        fetch(fi, fc);
+        prep();
+        put_kbar();
+        advance();
+        if (fi < a.items) fetch(fi, fc);
+    }
     for (int item = blockIdx.x; alive && item < a.items; item += gridDim.x) {
         const int b = item / a.Hv, h = item - b * a.Hv;
         float *Sg = a.states + (size_t)item * kN;
@@ -199,48 +258,9 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
         tc::wait_st();
         for (int t0 = 0; alive && t0 < a.T; t0 += C) {
             const int n = min(C, a.T - t0);               // tokens in this chunk (ragged tail)
+            fence_async_smem();                           // this chunk's operands visible to the tensor cores
             tc::fence_before();
             __syncthreads();                              // the previous chunk is done with every buffer
-            // Cumulative gates g_t per key channel (multiplied in token order) and beta.
-            if (tid < 128) {
-                float g = 1.f;
-#pragma unroll
-                for (int t = 0; t < C; t++) {
-                    g = fmaxf(g * dg[t], 1e-30f);         // keeps K / g finite
-                    G[t * 128 + tid] = g;
-                }
-            } else if (tid < 128 + C) {
-                bet[tid - 128] = bt;
-            }
-            __syncthreads();
-            // Element-wise: V, and the split operands [K~ ; Q~], K^ and K_bar^T,
-            // four consecutive K elements per store.
-            {
-                const int c4 = 4 * cq;
-                const float4 gC = *(const float4 *)&G[(C - 1) * 128 + c4];
-                float kb[4][4];                               // K_bar^T: [channel][token]
-#pragma unroll
-                for (int m = 0; m < 4; m++) {
-                    const int t = 4 * tq + m;
-                    const float4 g = *(const float4 *)&G[t * 128 + c4];
-                    const float4 rg = make_float4(__fdividef(1.0f, g.x), __fdividef(1.0f, g.y),   // within 2 ulp
-                                                  __fdividef(1.0f, g.z), __fdividef(1.0f, g.w));
-                    *(float4 *)&V[t * 128 + c4] = vv[m];
-                    put_split4(B1h, B1l, core_off(t, c4, kSbo128), mul4(g, kv[m]));        // K~
-                    put_split4(B1h, B1l, core_off(C + t, c4, kSbo128), mul4(g, qv[m]));    // Q~
-                    put_split4(B3h, B3l, core_off(t, c4, kSbo128), mul4(kv[m], rg));       // K^
-                    kb[0][m] = kv[m].x * (gC.x * rg.x);
-                    kb[1][m] = kv[m].y * (gC.y * rg.y);
-                    kb[2][m] = kv[m].z * (gC.z * rg.z);
-                    kb[3][m] = kv[m].w * (gC.w * rg.w);
-                }
-#pragma unroll
-                for (int e = 0; e < 4; e++)
-                    put_split4(B2h, B2l, core_off(c4 + e, 4 * tq, kSbo32),
-                               make_float4(kb[e][0], kb[e][1], kb[e][2], kb[e][3]));
-            }
-            fence_async_smem();                           // operands visible to the tensor cores
-            __syncthreads();
             // P0: [K~ ; Q~] K^T into columns [448, 480); P1: [K~ S_0 ; Q~ S_0]^T into [384, 448).
             if (tid == 0) {
                 tc::fence_after();
@@ -338,18 +358,19 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(Args a) {
                 tc::commit(bar);
             }
             __syncwarp();
-            {   // the next chunk's operands: this item's next chunk or the next item's first
-                int ni = item, nt = t0 + C;
-                if (nt >= a.T) {
-                    ni += gridDim.x;
-                    nt = 0;
-                }
-                if (ni < a.items) fetch(ni, nt);
+            // While P2 and P3 run: the next chunk's operands (this item's next
+            // chunk or the next item's first), and the inputs of the one after.
+            const bool more = fi < a.items;
+            if (more) {
+                prep();
+                advance();
+                if (fi < a.items) fetch(fi, fc);
             }
             if (!wait_mma()) {
                 alive = false;
                 break;
             }
+            if (more) put_kbar();                         // P2 is done with K_bar^T
             // Outputs: tokens 16 half .. 16 half + 15 of column j.
             {
                 float yv[16];
