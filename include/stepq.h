@@ -44,7 +44,7 @@ typedef enum {
     STEPQ_ERR_ALIGN = 4,        /* a buffer not aligned as documented */
     STEPQ_ERR_CUDA = 5,         /* a CUDA runtime call failed */
     STEPQ_ERR_BUDGET = 6,       /* the candidates cannot meet the bit budget */
-    STEPQ_ERR_UNSUPPORTED = 7,  /* a configuration this build does not implement */
+    STEPQ_ERR_UNSUPPORTED = 7,  /* a configuration the library does not implement */
     STEPQ_ERR_TIMEOUT = 8       /* a bounded device-side wait gave up (device-detected) */
 } stepq_status;
 
