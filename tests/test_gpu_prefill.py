@@ -52,6 +52,27 @@ def test_prefill_matches_recurrence(torch, name, T):
     assert np.abs(S_g - S_o).max() <= 1e-4 * np.abs(S_o).max()
 
 
+@pytest.mark.parametrize("name,B,T", [("gqa", 10, 45), ("channel", 6, 33)])
+def test_prefill_several_items_per_cta(torch, name, B, T):
+    """More (slot, head) items than SMs, so that each persistent CTA prepares the
+    next item's first chunk while the previous item's last chunk finishes; the
+    ragged tails end every item."""
+    wl = W.WORKLOADS[name]
+    cfg = A.Config.from_workload(wl)
+    assert B * wl.hv > torch.cuda.get_device_properties(0).multi_processor_count
+    S0 = O.warmup_states(wl, 0, B)
+    q, k, v, beta, gate = _tokens(wl, B, T)
+    S_o, y_o = _reference(S0, q, k, v, beta, gate)
+    S_d, q_d, k_d, v_d, b_d, g_d = to_dev(S0, q, k, v, beta, gate)
+    y_d = torch.empty((B, T, wl.hv, 128), dtype=torch.float32, device="cuda")
+    A.stepq_prefill_fp32(cfg, S_d, q_d, k_d, v_d, b_d, g_d, y_d)
+    y_g, S_g = y_d.cpu().numpy(), S_d.cpu().numpy()
+    rel = np.linalg.norm(y_g - y_o, axis=-1) / np.maximum(np.linalg.norm(y_o, axis=-1), 1e-30)
+    assert rel.max() <= 1e-4, rel.max()
+    assert np.abs(S_g - S_o).max() <= 1e-4 * np.abs(S_o).max()
+    assert A.stepq_device_error() == 0
+
+
 def test_prefill_empty_and_identity(torch):
     """T = 0 is a no-op; beta = 0 with gate 1 leaves the state unchanged."""
     wl = W.WORKLOADS["tiny"]
