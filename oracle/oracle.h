@@ -18,9 +18,10 @@
  *
  * Parity pins: every function here is pinned by tests under tests/ (closed
  * forms, identities of Sec. 2.1 / Prop. 1 / App. B.1 / App. B.3, brute force on
- * tiny inputs, the byte counts of App. D). Exact fitted scale values have no
- * closed form in the paper ("parity unpinned" for the column-fit values
- * themselves; their optimality for fixed codes is pinned instead).
+ * tiny inputs, the byte counts of App. D). The paper prints no fitted scale
+ * value; the fit is pinned step by step (the smallest clip-free column start,
+ * nearest codes, the fixed-code update as the 1-D minimiser of the weighted
+ * error, the row factors' scaling laws).
  */
 #ifndef STEPQ_ORACLE_H
 #define STEPQ_ORACLE_H

@@ -246,6 +246,11 @@ def test_fit_starts_clip_free_and_takes_one_update(oracle, rng, unit):
     Xd = X.astype(np.float64)
     start = (np.abs(Xd[nonpiv]) / (r * zs * qm)[nonpiv, None]).max(axis=0)
     assert np.allclose(c0, np.clip(start, 2.0 ** -14, 65504.0), rtol=1e-6)
+    # the smallest such scale: slightly below it some integer row of every
+    # column needs a code beyond qmax
+    below = Xd[nonpiv] / (r * zs)[nonpiv, None] / (c0.astype(np.float64) * (1 - 1e-5))[None, :]
+    inside = c0 > 2.0 ** -14
+    assert np.all((np.abs(below) > qm[nonpiv, None]).any(axis=0)[inside])
     r1, c1, z1 = oracle.fit_debug(X, unit, rb, w, 1)
     assert np.array_equal(r1, r)
     t = Xd[nonpiv] / (r * zs)[nonpiv, None] / c0.astype(np.float64)[None, :]
