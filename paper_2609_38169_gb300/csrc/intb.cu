@@ -5,7 +5,9 @@
 //
 // Tile mapping: warp w owns key rows 16w..16w+15, lane l the value columns
 // 4l..4l+3; a lane's 4 codes of a row are one word (8-bit), three bytes at
-// byte 3l (6-bit) or a half-word (4-bit).
+// byte 3l (6-bit) or a half-word (4-bit). A thread holds its 16 rows as eight
+// row pairs per column, each pair one packed f32x2 register, so one 128-bit
+// load of a per-row constant serves two pairs.
 // Per row the tile holds Z = q with X_ij = a_i Z_ij, a_i = s_i d_i (d_i the
 // gate), so the decode is the code itself. Every column reduction needs one
 // cross-warp step; the row absmax is a warp reduce-scatter.
@@ -22,23 +24,26 @@ namespace ib {
 constexpr int kOffBars = 0;                            // uint64 [8]
 constexpr int kOffRed = 64;                            // float [2][8][128]: retrieval, readout
 constexpr int kOffColD = kOffRed + 2 * 8 * 128 * 4;    // float [128] delta_j
-constexpr int kOffRows = kOffColD + 512;               // float4 [3][128] per-row constants
-constexpr int kOffStages = (kOffRows + 3 * 128 * 16 + 127) / 128 * 128;
+constexpr int kOffRows = kOffColD + 512;               // float [6][128] per-row constants
+constexpr int kOffStages = (kOffRows + 6 * 128 * 4 + 127) / 128 * 128;
 
 struct Smem {
     uint64_t *bars;
     float *red, *colD;
-    float4 *rowK;   // (kappa, kappa, beta k / a, beta k / a), kappa = k a
-    float4 *rowQ;   // (q a, q a, a, a)
-    float4 *rowT;   // (a / s_new, a / s_new, clamp limit or 0, -)
+    // per-row constants: kappa = k a, beta k / a, q a, a, a / s_new and the
+    // clamp limit (q_b where the new scale was capped, else no limit)
+    float *rKap, *rBkp, *rQa, *rA, *rTs, *rLim;
     uint8_t *stages;
     __device__ __forceinline__ explicit Smem(uint8_t *s) {
         bars = (uint64_t *)(s + kOffBars);
         red = (float *)(s + kOffRed);
         colD = (float *)(s + kOffColD);
-        rowK = (float4 *)(s + kOffRows);
-        rowQ = rowK + 128;
-        rowT = rowK + 256;
+        rKap = (float *)(s + kOffRows);
+        rBkp = rKap + 128;
+        rQa = rKap + 256;
+        rA = rKap + 384;
+        rTs = rKap + 512;
+        rLim = rKap + 640;
         stages = s + kOffStages;
     }
 };
@@ -80,10 +85,11 @@ struct T {
     __device__ __forceinline__ int row(int r) const { return 16 * w + r; }
 };
 
-__device__ __forceinline__ void row_dup(const float4 *v, int i, uint64_t &xx, uint64_t &zz) {
-    const uint4 q = *(const uint4 *)&v[i];
-    xx = u2pair(q.x, q.y);
-    zz = u2pair(q.z, q.w);
+// Row-pair constants (rows 4p, 4p+1) and (4p+2, 4p+3) of the warp's band.
+__device__ __forceinline__ void row_pairs(const float *v, const T &t, int p, uint64_t &lo, uint64_t &hi) {
+    const uint4 q = *(const uint4 *)&v[t.row(4 * p)];
+    lo = u2pair(q.x, q.y);
+    hi = u2pair(q.z, q.w);
 }
 
 // Warp reduce-scatter of 16 per-row maxima (as warp_row_sums, with max).
@@ -116,35 +122,27 @@ __device__ __forceinline__ float warp_row_max(float (&v)[16], int l, int &row_ou
     return a1;
 }
 
+// The lane's 4 codes of a row as the bit patterns 1.5*2^23 + u (one logic
+// op or byte permute each).
 template <int B>
-__device__ __forceinline__ void decode_row(const uint8_t *row, int l, uint64_t &x0, uint64_t &x1) {
-    uint32_t f0, f1, f2, f3;
+__device__ __forceinline__ void row_codes(const uint8_t *row, int l, uint32_t (&f)[4]) {
     if (B == 8) {
         const uint32_t w = ((const uint32_t *)row)[l];
-        f0 = __byte_perm(w, kMagicBits, 0x7650);
-        f1 = __byte_perm(w, kMagicBits, 0x7651);
-        f2 = __byte_perm(w, kMagicBits, 0x7652);
-        f3 = __byte_perm(w, kMagicBits, 0x7653);
+#pragma unroll
+        for (int c = 0; c < 4; c++) f[c] = __byte_perm(w, kMagicBits, 0x7650u + (uint32_t)c);
     } else if (B == 6) {
         // 24 bits at bit 24 l: a funnel shift of the two words that hold them
         // (the last lane's upper word is clamped into the row; it is unused).
         const uint32_t *wd = (const uint32_t *)row;
         const int wi = (3 * l) >> 2;
         const uint32_t x = __funnelshift_r(wd[wi], wd[min(wi + 1, 23)], 8 * ((3 * l) & 3));
-        f0 = and_or(x, 0x3Fu, kMagicBits);
-        f1 = and_or(x >> 6, 0x3Fu, kMagicBits);
-        f2 = and_or(x >> 12, 0x3Fu, kMagicBits);
-        f3 = and_or(x >> 18, 0x3Fu, kMagicBits);
+#pragma unroll
+        for (int c = 0; c < 4; c++) f[c] = and_or(x >> (6 * c), 0x3Fu, kMagicBits);
     } else {
         const uint32_t x = ((const uint16_t *)row)[l];
-        f0 = and_or(x, 0xFu, kMagicBits);
-        f1 = and_or(x >> 4, 0xFu, kMagicBits);
-        f2 = and_or(x >> 8, 0xFu, kMagicBits);
-        f3 = and_or(x >> 12, 0xFu, kMagicBits);
+#pragma unroll
+        for (int c = 0; c < 4; c++) f[c] = and_or(x >> (4 * c), 0xFu, kMagicBits);
     }
-    const uint64_t off = f2s(-(kMagic + (float)(1 << (B - 1))));
-    x0 = fadd2(u2pair(f0, f1), off);
-    x1 = fadd2(u2pair(f2, f3), off);
 }
 
 template <int B>
@@ -180,28 +178,40 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         const int i = t.row(t.l);
         const float dg = per_row ? st.gate[i] : gate_s;
         const float a = fmaxf(f16_val(page_s[i]) * dg, 1e-30f);
-        const float ki = st.k[i], kap = ki * a, bkp = __fdividef(beta * ki, a), qa = st.q[i] * a;
-        S.rowK[i] = make_float4(kap, kap, bkp, bkp);
-        S.rowQ[i] = make_float4(qa, qa, a, a);
+        const float ki = st.k[i];
+        S.rKap[i] = ki * a;
+        S.rBkp[i] = __fdividef(beta * ki, a);
+        S.rQa[i] = st.q[i] * a;
+        S.rA[i] = a;
     }
-    uint64_t x2[16][2];
+    // Z = q: rows 2m, 2m+1 of column 4l + c as one pair
+    uint64_t x2[8][4];
+    {
+        const uint64_t off = f2s(-(kMagic + (float)(1 << (B - 1))));
 #pragma unroll
-    for (int r = 0; r < 16; r++) decode_row<B>(codes + t.row(r) * 16 * B, t.l, x2[r][0], x2[r][1]);
+        for (int m = 0; m < 8; m++) {
+            uint32_t f0[4], f1[4];
+            row_codes<B>(codes + t.row(2 * m) * 16 * B, t.l, f0);
+            row_codes<B>(codes + t.row(2 * m + 1) * 16 * B, t.l, f1);
+#pragma unroll
+            for (int c = 0; c < 4; c++) x2[m][c] = fadd2(u2pair(f0[c], f1[c]), off);
+        }
+    }
     __syncwarp();
     {
-        uint64_t ua[2] = {0, 0}, ub[2] = {0, 0};
+        uint64_t ua[4] = {0, 0, 0, 0};
 #pragma unroll
-        for (int r = 0; r < 16; r += 2) {
-            uint64_t k0, k1, z;
-            row_dup(S.rowK, t.row(r), k0, z);
-            row_dup(S.rowK, t.row(r + 1), k1, z);
-            ua[0] = ffma2(k0, x2[r][0], ua[0]);
-            ua[1] = ffma2(k0, x2[r][1], ua[1]);
-            ub[0] = ffma2(k1, x2[r + 1][0], ub[0]);
-            ub[1] = ffma2(k1, x2[r + 1][1], ub[1]);
+        for (int p = 0; p < 4; p++) {
+            uint64_t klo, khi;
+            row_pairs(S.rKap, t, p, klo, khi);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                ua[c] = ffma2(klo, x2[2 * p][c], ua[c]);
+                ua[c] = ffma2(khi, x2[2 * p + 1][c], ua[c]);
+            }
         }
-        const uint64_t s0 = fadd2(ua[0], ub[0]), s1 = fadd2(ua[1], ub[1]);
-        *(float4 *)&S.red[t.w * 128 + 4 * t.l] = make_float4(f2lo(s0), f2hi(s0), f2lo(s1), f2hi(s1));
+        *(float4 *)&S.red[t.w * 128 + 4 * t.l] =
+            make_float4(pair_sum(ua[0]), pair_sum(ua[1]), pair_sum(ua[2]), pair_sum(ua[3]));
     }
     if (__syncthreads_or(!ok)) return false;
     if (t.tid < 128) {
@@ -215,28 +225,32 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     // Z += (beta k_i / a_i) delta_j; readout partials; per-row max |Z|.
     float rm[16];
     {
-        const uint4 dq = *(const uint4 *)&S.colD[4 * t.l];
-        const uint64_t d01 = u2pair(dq.x, dq.y), d23 = u2pair(dq.z, dq.w);
-        uint64_t ya[2] = {0, 0}, yb[2] = {0, 0};
+        const float4 dq = *(const float4 *)&S.colD[4 * t.l];
+        const uint64_t dl[4] = {f2s(dq.x), f2s(dq.y), f2s(dq.z), f2s(dq.w)};
+        uint64_t ya[4] = {0, 0, 0, 0};
 #pragma unroll
-        for (int r = 0; r < 16; r++) {
-            uint64_t z, bk, qa;
-            row_dup(S.rowK, t.row(r), z, bk);
-            row_dup(S.rowQ, t.row(r), qa, z);
-            x2[r][0] = ffma2(bk, d01, x2[r][0]);
-            x2[r][1] = ffma2(bk, d23, x2[r][1]);
-            if (r & 1) {
-                yb[0] = ffma2(qa, x2[r][0], yb[0]);
-                yb[1] = ffma2(qa, x2[r][1], yb[1]);
-            } else {
-                ya[0] = ffma2(qa, x2[r][0], ya[0]);
-                ya[1] = ffma2(qa, x2[r][1], ya[1]);
+        for (int p = 0; p < 4; p++) {
+            uint64_t blo, bhi, qlo, qhi;
+            row_pairs(S.rBkp, t, p, blo, bhi);
+            row_pairs(S.rQa, t, p, qlo, qhi);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                x2[2 * p][c] = ffma2(blo, dl[c], x2[2 * p][c]);
+                x2[2 * p + 1][c] = ffma2(bhi, dl[c], x2[2 * p + 1][c]);
+                ya[c] = ffma2(qlo, x2[2 * p][c], ya[c]);
+                ya[c] = ffma2(qhi, x2[2 * p + 1][c], ya[c]);
             }
-            rm[r] = fmax3(fmax3(0.f, fabsf(f2lo(x2[r][0])), fabsf(f2hi(x2[r][0]))),
-                          fabsf(f2lo(x2[r][1])), fabsf(f2hi(x2[r][1])));
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                const uint64_t(&xm)[4] = x2[2 * p + h];
+                rm[4 * p + 2 * h] = fmax3(fmax3(0.f, fabsf(f2lo(xm[0])), fabsf(f2lo(xm[1]))),
+                                          fabsf(f2lo(xm[2])), fabsf(f2lo(xm[3])));
+                rm[4 * p + 2 * h + 1] = fmax3(fmax3(0.f, fabsf(f2hi(xm[0])), fabsf(f2hi(xm[1]))),
+                                              fabsf(f2hi(xm[2])), fabsf(f2hi(xm[3])));
+            }
         }
-        const uint64_t s0 = fadd2(ya[0], yb[0]), s1 = fadd2(ya[1], yb[1]);
-        *(float4 *)&S.red[(8 + t.w) * 128 + 4 * t.l] = make_float4(f2lo(s0), f2hi(s0), f2lo(s1), f2hi(s1));
+        *(float4 *)&S.red[(8 + t.w) * 128 + 4 * t.l] =
+            make_float4(pair_sum(ya[0]), pair_sum(ya[1]), pair_sum(ya[2]), pair_sum(ya[3]));
     }
     // Row scale s_i = fp16(clamp(absmax_i / q_b)), absmax_i = a_i max_j |Z_ij|.
     {
@@ -244,11 +258,11 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         const float zmax = warp_row_max(rm, t.l, rr);
         const int i = t.row(rr);
         if ((t.l & 1) == 0) {
-            const float a = S.rowQ[i].z;
+            const float a = S.rA[i];
             const float q = __fdiv_rn(a * zmax, (float)qm);
             const float s = __half2float(__float2half_rn(fminf(fmaxf(q, kF16Min), kF16Max)));
-            const float ts = a * __frcp_rn(s);                // t = Z (a / s)
-            S.rowT[i] = make_float4(ts, ts, q > kF16Max ? (float)qm : 0.f, 0.f);
+            S.rTs[i] = a * __frcp_rn(s);                      // t = Z (a / s)
+            S.rLim[i] = q > kF16Max ? (float)qm : 3.0e38f;
             page_s[i] = f16_bits(s);
         }
     }
@@ -262,18 +276,28 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
     // Codes rne(X / s_i) (clamped only where the scale was capped), in place.
     const uint64_t mb = f2s(kMagic + (float)(1 << (B - 1)));
 #pragma unroll
-    for (int r = 0; r < 16; r++) {
-        uint64_t ts, lim;
-        row_dup(S.rowT, t.row(r), ts, lim);
-        uint64_t t0 = fmul2(x2[r][0], ts), t1 = fmul2(x2[r][1], ts);
-        const float cl = f2lo(lim);
-        if (cl != 0.f) {
-            t0 = clamp2(t0, cl);
-            t1 = clamp2(t1, cl);
+    for (int p = 0; p < 4; p++) {
+        uint64_t tlo, thi, llo, lhi;
+        row_pairs(S.rTs, t, p, tlo, thi);
+        row_pairs(S.rLim, t, p, llo, lhi);
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+            const int m = 2 * p + h;
+            const uint64_t ts = h ? thi : tlo, lim = h ? lhi : llo;
+            const bool capped = fminf(f2lo(lim), f2hi(lim)) < 1.0e38f;   // uniform across the warp
+            uint32_t f0[4], f1[4];
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                uint64_t tt = fmul2(x2[m][c], ts);
+                if (capped) tt = f2(fminf(fmaxf(f2lo(tt), -f2lo(lim)), f2lo(lim)),
+                                    fminf(fmaxf(f2hi(tt), -f2hi(lim)), f2hi(lim)));
+                const uint64_t u = fadd2(tt, mb);
+                f0[c] = (uint32_t)u;
+                f1[c] = (uint32_t)(u >> 32);
+            }
+            store_row<B>(codes + t.row(2 * m) * 16 * B, t.l, f0[0], f0[1], f0[2], f0[3]);
+            store_row<B>(codes + t.row(2 * m + 1) * 16 * B, t.l, f1[0], f1[1], f1[2], f1[3]);
         }
-        const uint64_t u0 = fadd2(t0, mb), u1 = fadd2(t1, mb);
-        store_row<B>(codes + t.row(r) * 16 * B, t.l, (uint32_t)u0, (uint32_t)(u0 >> 32), (uint32_t)u1,
-                     (uint32_t)(u1 >> 32));
     }
     return true;
 }
