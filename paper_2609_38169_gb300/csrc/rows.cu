@@ -349,11 +349,13 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         const int sl = t.row(t.l);                         // stored slot; i = its key row
         // The row table arrives with the page; a stage whose copies did not
         // complete still holds whatever it held, and the first CTA barrier ends
-        // the item then. Offset and width are capped first so that the page reads
-        // before that barrier stay inside the stage whatever the table holds.
+        // the item then. Offset and width are capped first, and the offset
+        // rounded down to the 32 bytes every row start has, so that the page
+        // reads before that barrier stay inside the stage and aligned whatever
+        // the table holds.
         const uint32_t raw = st.slot[sl];
         const uint32_t region = (uint32_t)((const uint8_t *)st.q - st.page);
-        const uint32_t off = min(raw & 0xFFFFu, region), bw = min((raw >> 16) & 0xFFu, (uint32_t)kPivot);
+        const uint32_t off = min(raw & 0xFFFFu, region) & ~31u, bw = min((raw >> 16) & 0xFFu, (uint32_t)kPivot);
         const uint32_t info = off | (bw << 16) | (raw & 0xFF000000u);
         const int b = (int)bw, i = (int)(info >> 24);
         const float dg = st.gate[i];
