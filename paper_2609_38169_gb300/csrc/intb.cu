@@ -166,6 +166,37 @@ __device__ __forceinline__ void store_row(uint8_t *row, int l, uint32_t f0, uint
     }
 }
 
+// Codes rne(X / s_i) of the warp's 16 rows, written in place; CLIP clamps each
+// row to its limit (q_b where the row's scale was capped, else none).
+template <int B, bool CLIP>
+__device__ __forceinline__ void requant_rows(const T &t, const Smem &S, uint8_t *codes,
+                                             const uint64_t (&x2)[8][4]) {
+    const uint64_t mb = f2s(kMagic + (float)(1 << (B - 1)));
+#pragma unroll
+    for (int p = 0; p < 4; p++) {
+        uint64_t tlo, thi, llo = 0, lhi = 0;
+        row_pairs(S.rTs, t, p, tlo, thi);
+        if (CLIP) row_pairs(S.rLim, t, p, llo, lhi);
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+            const int m = 2 * p + h;
+            const uint64_t ts = h ? thi : tlo, lim = h ? lhi : llo;
+            uint32_t f0[4], f1[4];
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                uint64_t tt = fmul2(x2[m][c], ts);
+                if (CLIP) tt = f2(fminf(fmaxf(f2lo(tt), -f2lo(lim)), f2lo(lim)),
+                                  fminf(fmaxf(f2hi(tt), -f2hi(lim)), f2hi(lim)));
+                const uint64_t u = fadd2(tt, mb);
+                f0[c] = (uint32_t)u;
+                f1[c] = (uint32_t)(u >> 32);
+            }
+            store_row<B>(codes + t.row(2 * m) * 16 * B, t.l, f0[0], f0[1], f0[2], f0[3]);
+            store_row<B>(codes + t.row(2 * m + 1) * 16 * B, t.l, f1[0], f1[1], f1[2], f1[3]);
+        }
+    }
+}
+
 // One INT-b decode step of a head page staged in shared memory.
 template <int B, class Refill>
 __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Stage &st, float gate_s,
@@ -252,14 +283,17 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         *(float4 *)&S.red[(8 + t.w) * 128 + 4 * t.l] =
             make_float4(pair_sum(ya[0]), pair_sum(ya[1]), pair_sum(ya[2]), pair_sum(ya[3]));
     }
-    // Row scale s_i = fp16(clamp(absmax_i / q_b)), absmax_i = a_i max_j |Z_ij|.
+    // Row scale s_i = fp16(clamp(absmax_i / q_b)), absmax_i = a_i max_j |Z_ij|
+    // (lanes l and l ^ 1 hold the same row; the even one writes it).
+    bool capped;                                            // a row of the warp's band was capped
     {
         int rr;
         const float zmax = warp_row_max(rm, t.l, rr);
         const int i = t.row(rr);
+        const float a = S.rA[i];
+        const float q = __fdiv_rn(a * zmax, (float)qm);
+        capped = __any_sync(0xffffffffu, q > kF16Max);
         if ((t.l & 1) == 0) {
-            const float a = S.rA[i];
-            const float q = __fdiv_rn(a * zmax, (float)qm);
             const float s = __half2float(__float2half_rn(fminf(fmaxf(q, kF16Min), kF16Max)));
             S.rTs[i] = a * __frcp_rn(s);                      // t = Z (a / s)
             S.rLim[i] = q > kF16Max ? (float)qm : 3.0e38f;
@@ -273,32 +307,9 @@ __device__ __forceinline__ bool decode_item(const T &t, const Smem &S, const Sta
         for (int wv = 1; wv < 8; wv++) s += S.red[(8 + wv) * 128 + t.tid];
         y_out[t.tid] = s;
     }
-    // Codes rne(X / s_i) (clamped only where the scale was capped), in place.
-    const uint64_t mb = f2s(kMagic + (float)(1 << (B - 1)));
-#pragma unroll
-    for (int p = 0; p < 4; p++) {
-        uint64_t tlo, thi, llo, lhi;
-        row_pairs(S.rTs, t, p, tlo, thi);
-        row_pairs(S.rLim, t, p, llo, lhi);
-#pragma unroll
-        for (int h = 0; h < 2; h++) {
-            const int m = 2 * p + h;
-            const uint64_t ts = h ? thi : tlo, lim = h ? lhi : llo;
-            const bool capped = fminf(f2lo(lim), f2hi(lim)) < 1.0e38f;   // uniform across the warp
-            uint32_t f0[4], f1[4];
-#pragma unroll
-            for (int c = 0; c < 4; c++) {
-                uint64_t tt = fmul2(x2[m][c], ts);
-                if (capped) tt = f2(fminf(fmaxf(f2lo(tt), -f2lo(lim)), f2lo(lim)),
-                                    fminf(fmaxf(f2hi(tt), -f2hi(lim)), f2hi(lim)));
-                const uint64_t u = fadd2(tt, mb);
-                f0[c] = (uint32_t)u;
-                f1[c] = (uint32_t)(u >> 32);
-            }
-            store_row<B>(codes + t.row(2 * m) * 16 * B, t.l, f0[0], f0[1], f0[2], f0[3]);
-            store_row<B>(codes + t.row(2 * m + 1) * 16 * B, t.l, f1[0], f1[1], f1[2], f1[3]);
-        }
-    }
+    // Codes rne(X / s_i) (clamped only in warps with a capped row), in place.
+    if (capped) requant_rows<B, true>(t, S, codes, x2);
+    else requant_rows<B, false>(t, S, codes, x2);
     return true;
 }
 
