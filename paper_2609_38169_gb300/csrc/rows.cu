@@ -137,22 +137,15 @@ __device__ __forceinline__ uint32_t lane_segment(const uint8_t *row, int b, int 
     return __funnelshift_r(wp[bit >> 5], wp[(bit >> 5) + 1], bit & 31);
 }
 
-// Write the lane's 4b-bit segment v (b in {2, 4, 6, 8}) into the row.
+// Write the lane's 4b-bit segment v (b in {2, 4, 6, 8}) into the row: b/2
+// bytes from byte l b/2, as byte stores under warp-uniform conditions (no
+// branches; the lanes never share a byte).
 __device__ __forceinline__ void store_segment(uint8_t *row, int b, int l, uint32_t v) {
-    if (b == 8) {
-        ((uint32_t *)row)[l] = v;
-    } else if (b == 4) {
-        ((uint16_t *)row)[l] = (uint16_t)v;
-    } else if (b == 2) {
-        row[l] = (uint8_t)v;
-    } else {
-        // 24 bits per lane, bytes 3l .. 3l + 2: one aligned 16-bit store and one
-        // byte store (which is which depends on l's parity)
-        const int odd = l & 1;
-        uint8_t *p = row + 3 * l;
-        *(uint16_t *)(p + odd) = (uint16_t)(odd ? v >> 8 : v);
-        p[odd ? 0 : 2] = (uint8_t)(odd ? v : v >> 16);
-    }
+    uint8_t *p = row + ((l * b) >> 1);
+    p[0] = (uint8_t)v;
+    if (b >= 4) p[1] = (uint8_t)(v >> 8);
+    if (b >= 6) p[2] = (uint8_t)(v >> 16);
+    if (b >= 8) p[3] = (uint8_t)(v >> 24);
 }
 
 // Sum over the 4 codes of a lane segment of (0x4B400000 << k b): what the
