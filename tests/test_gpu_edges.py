@@ -96,6 +96,61 @@ def test_degenerate_states(torch, name, kw):
     assert A.stepq_device_error() == 0
 
 
+@pytest.mark.parametrize("bits,name", [(8, "gqa"), (4, "channel")])
+def test_intb_degenerate_states(torch, bits, name):
+    """The INT-b comparison kernel on the same edge-case states: a zero state,
+    a huge one whose row scales are capped at 65504 (so the codes are clamped
+    to +-q_b, App. B.5), tiny ones and sparse outliers; teacher-forced against
+    the oracle for 2 steps."""
+    wl = W.WORKLOADS[name].replace(pool_slots=4)
+    cfg = A.Config.from_workload(wl)
+    mp = W.model_params(wl)
+    S = _degenerate_states(wl)
+    B = S.shape[0]
+    slots = np.arange(B, dtype=np.int32)[::-1].copy()
+    stride = A.stepq_intb_slot_bytes(cfg, bits)
+    hb = O.intb_head_bytes(bits)
+    pool_o = np.zeros(wl.pool_slots * stride, np.uint8)
+    for b in range(B):
+        for h in range(wl.hv):
+            base = int(slots[b]) * stride + h * hb
+            pool_o[base:base + hb] = O.intb_encode_head(S[b, h], bits)
+    (slots_d,) = to_dev(slots)
+    pool_d = torch.zeros(wl.pool_slots * stride, dtype=torch.uint8, device="cuda")
+    t = Tally()
+    for step in range(2):
+        inp = W.step_inputs(wl, mp, W.STREAM_DECODE, step, 0, batch=B)
+        pool_d.copy_(torch.from_numpy(pool_o))
+        q, k, v, beta, gate = to_dev(inp.q, inp.k, inp.v, inp.beta, inp.gate)
+        y_d = torch.empty((B, wl.hv, 128), dtype=torch.float32, device="cuda")
+        A.stepq_intb_decode_step(cfg, bits, 0, pool_d, slots_d, q, k, v, beta, gate, y_d)
+        y_o = O.intb_pool_step(bits, wl.hk, wl.hv, wl.gate_per_row, 0, stride, pool_o, slots, inp)
+        assert np.isfinite(y_d.cpu().numpy()).all()
+        compare_y(t, y_d.cpu().numpy(), y_o)
+        got = pool_d.cpu().numpy()
+        for b in range(B):
+            for h in range(wl.hv):
+                base = int(slots[b]) * stride + h * hb
+                sg = got[base:base + 256].view(np.uint16)
+                so = pool_o[base:base + 256].view(np.uint16)
+                t.scales += 128
+                t.scale_diff += int(np.count_nonzero(sg != so))
+                cg = np.unpackbits(got[base + 256:base + hb], bitorder="little")
+                co = np.unpackbits(pool_o[base + 256:base + hb], bitorder="little")
+                ug = (cg.reshape(-1, bits) * (1 << np.arange(bits))).sum(1)
+                uo = (co.reshape(-1, bits) * (1 << np.arange(bits))).sum(1)
+                t.elems += ug.size
+                t.code_diff += int(np.count_nonzero(ug != uo))
+                t.code_maxdiff = max(t.code_maxdiff, int(np.abs(ug - uo).max()))
+    # the huge slot's rows keep scales capped at FP16 65504 (0x7BFF) through the
+    # step, so the clamped code path ran
+    capped = got[int(slots[1]) * stride:][:256].view(np.uint16)
+    assert (capped == 0x7BFF).any()
+    print(bits, name, t.summary())
+    t.check()
+    assert A.stepq_device_error() == 0
+
+
 def test_largest_head_count(torch):
     """256 value heads (64 key heads) per layer, the most one launch takes."""
     wl = W.WORKLOADS["gqa"].replace(name="maxheads", hk=64, hv=256, batch=2, pool_slots=4, n_pivots=5)
